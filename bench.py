@@ -1,0 +1,375 @@
+#!/usr/bin/env python3
+"""Benchmark of the FlashVLA streaming action-decode step on GB300 (libfva).
+
+Default workload: the pi0.5-shaped expert (18 layers, width 1024, 8 query heads /
+1 KV head of 256, MLP 4096, action dim 32) with a 560-token prefix and a K=10 x
+H=50 buffer at batch 1, synthetic seeded inputs.  A step is one fva_step: one
+expert forward over the whole buffer, the per-chunk Euler update, emit, roll and
+tail push.
+
+Prints ONE JSON line (rank 0):
+  value       steps/s with every input resident in HBM (CUDA-graph replay through
+              fva_step, CUDA events on the launching stream, max over ranks);
+  e2e         the same through the C ABI with the buffer copied in from pinned host
+              memory and the emitted chunk copied back every step;
+  roofline    the dominant kernel (largest share of a kernel-by-kernel profiled
+              step) against the measured peak of its binding resource;
+  step_roofline  the whole step against max(FLOPs / tensor peak, bytes / HBM peak);
+  cpu_baseline   the CPU oracle timed on this host on a bounded sample.
+Under torchrun every rank runs an independent replica (requests shard with no
+exchange); `value` counts the steps of all ranks.
+
+`--impl reference` times the CPU oracle instead (the reference arm).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads as WL  # noqa: E402
+
+METRIC = "streaming decode steps/s (executable chunks/s) at batch 1; µs/step; % of roofline"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ---------------------------------------------------------------------------
+# algorithmic work per kernel launch (FLOPs, bytes)
+# ---------------------------------------------------------------------------
+
+def kernel_costs(wl, B):
+    """Algorithmic FLOPs and DRAM bytes of one launch of each kernel kind (bf16
+    weights, bf16 activations, fp32 residual stream)."""
+    W, F, Dq, dh, nq, K, H, A = (wl.width, wl.mlp_dim, wl.n_q_heads * wl.head_dim,
+                                 wl.head_dim, wl.n_q_heads, wl.n_chunks, wl.chunk_tokens,
+                                 wl.action_dim)
+    T = K * H
+    M = B * T
+    BK = B * K
+    L = wl.n_layers
+    Nqkv = Dq + 2 * dh
+    Nmod = L * 6 * W + 2 * W
+    P = wl.prefix_lens[:B]
+    pairs = sum(p * T + H * H * K * (K + 1) // 2 for p in P)
+    c = {}
+    c["qkv"] = (2.0 * M * W * Nqkv, 2.0 * (Nqkv * W + M * W + M * Nqkv))
+    c["out_proj"] = (2.0 * M * Dq * W, 2.0 * (W * Dq + M * Dq) + 4.0 * M * W)
+    c["gate_up"] = (2.0 * M * W * 2 * F, 2.0 * (2 * F * W + M * W + M * F))
+    c["down"] = (2.0 * M * F * W, 2.0 * (W * F + M * F) + 4.0 * M * W)
+    c["attention"] = (4.0 * dh * nq * pairs, 2.0 * (sum(P) + B * T) * dh * 2 + 2.0 * 2 * M * Dq)
+    c["film"] = (2.0 * BK * W * Nmod, 2.0 * Nmod * W + 4.0 * BK * Nmod)
+    c["time_mlp"] = (2.0 * BK * W * W, 2.0 * W * W)
+    c["resid_norm"] = (0.0, 4.0 * M * W * 3 + 2.0 * M * W)
+    c["embed_norm"] = (2.0 * M * A * W, 4.0 * M * (A + W) + 2.0 * M * W)
+    c["final"] = (2.0 * M * W * A, 4.0 * M * W * 2 + 4.0 * M * A * 3)
+    c["timestep_embed"] = (0.0, 2.0 * BK * W)
+    return c
+
+
+def step_costs(wl, B):
+    """Whole-step algorithmic FLOPs and the HBM bytes that must be streamed (every
+    weight once + the prefix K/V of every layer)."""
+    L = wl.n_layers
+    c = kernel_costs(wl, B)
+    flops = L * sum(c[k][0] for k in ("qkv", "out_proj", "gate_up", "down", "attention"))
+    flops += c["film"][0] + 2 * c["time_mlp"][0] + c["embed_norm"][0] + c["final"][0]
+    W, F, Dq, dh, A = wl.width, wl.mlp_dim, wl.n_q_heads * wl.head_dim, wl.head_dim, wl.action_dim
+    wbytes = 2.0 * L * ((Dq + 2 * dh) * W + W * Dq + 2 * F * W + W * F)
+    wbytes += 2.0 * (L * 6 * W + 2 * W) * W + 2.0 * 2 * W * W + 4.0 * 2 * A * W
+    kv = 2.0 * L * sum(wl.prefix_lens[:B]) * dh * 2
+    return flops, wbytes + kv
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.tmp = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.tmp, stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.tmp.flush()
+        with open(self.tmp.name) as f:
+            rows = [r.split(",") for r in f.read().strip().splitlines() if r.strip()]
+        os.unlink(self.tmp.name)
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            r = [x.strip() for x in r]
+            if len(r) < 7:
+                continue
+            try:
+                sm.append(float(r[0]))
+                mx = float(r[1])
+            except ValueError:
+                continue
+            for n, v in zip(names, r[3:7]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def gpu_index_for(local_rank: int) -> int:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [v.strip() for v in vis.split(",") if v.strip()]
+        if local_rank < len(ids) and ids[local_rank].isdigit():
+            return int(ids[local_rank])
+    return local_rank
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (baseline / reference arm)
+# ---------------------------------------------------------------------------
+
+def time_oracle(wl, w, pre, buf, tau, budget_s: float, max_steps: int):
+    import oracle
+    fresh = np.zeros((wl.batch, wl.chunk_tokens, wl.action_dim), np.float32)
+    t0 = time.perf_counter()
+    oracle.stream_step(w, wl.as_config(), buf, tau, pre, fresh)
+    first = time.perf_counter() - t0
+    n = int(max(1, min(max_steps, budget_s // max(first, 1e-9))))
+    t0 = time.perf_counter()
+    for _ in range(n):
+        oracle.stream_step(w, wl.as_config(), buf, tau, pre, fresh)
+    dt = time.perf_counter() - t0
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    return n, dt, cores
+
+
+# ---------------------------------------------------------------------------
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=4000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", choices=["fva", "reference"], default="fva")
+    ap.add_argument("--workload", default="pi05_2view", choices=list(WL.standard_workloads()))
+    ap.add_argument("--profile-steps", type=int, default=20)
+    ap.add_argument("--cpu-budget", type=float, default=20.0,
+                    help="seconds of oracle work for the CPU baseline")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    wl = WL.standard_workloads()[args.workload]
+    peaks, peak_src = load_peaks()
+    cfg_json = {"workload": wl.name, "batch": wl.batch, "n_chunks": wl.n_chunks,
+                "chunk_tokens": wl.chunk_tokens, "prefix_tokens": wl.prefix_lens[:4],
+                "n_layers": wl.n_layers, "width": wl.width, "heads": f"{wl.n_q_heads}q/1kv",
+                "head_dim": wl.head_dim, "mlp_dim": wl.mlp_dim, "action_dim": wl.action_dim,
+                "parallelism": f"replicas x{args.gpus}" if args.gpus > 1 else "single GPU",
+                "l2": "no flush: every step streams ~0.87 GB of weights + prefix K/V > 129 MB L2",
+                "weights": "seeded N(0, 0.02), bf16"}
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        w = WL.make_weights(wl)
+        pre = WL.make_prefix_kv(wl)
+        buf, tau = WL.make_buffer(wl), WL.make_noise_levels(wl)
+        n, dt, cores = time_oracle(wl, w, pre, buf, tau, budget_s=60.0, max_steps=args.steps)
+        v = n / dt
+        line = {"metric": METRIC, "value": v, "unit": "steps/s", "impl": "reference",
+                "n_gpus": args.gpus, "steps": n, "warmup": 1, "ms_per_step": 1e3 * dt / n,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "f64", "data": "synthetic", "config": cfg_json,
+                "cpu_baseline": {"value": v, "unit": "steps/s", "cores": cores, "kind": "oracle",
+                                 "sample": f"{n} full oracle steps (of {args.steps} requested; "
+                                           "bounded to ~60 s of CPU work)"},
+                "e2e": {"value": v, "unit": "steps/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return 0
+
+    import torch
+    import paper_2608_27384_gb300 as fva
+    from paper_2608_27384_gb300.harness import Decoder
+
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", local_rank if world > 1 else 0)
+
+    w = WL.make_weights(wl)
+    pre = WL.make_prefix_kv(wl)
+    buf = WL.make_buffer(wl)
+    tau = WL.make_noise_levels(wl)
+    dec = Decoder(wl, WL.flat_weights(wl, w), pre)
+    h = dec.handle
+    B = wl.batch
+    stream = torch.cuda.Stream(device=dev)
+    d_buf = torch.from_numpy(buf).to(dev)
+    d_out = torch.empty((B, wl.chunk_tokens, wl.action_dim), device=dev)
+
+    def barrier():
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(x: float) -> float:
+        if dist is None:
+            return x
+        t = torch.tensor([x], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    # ---- device-resident timing: graph replay through fva_step
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            fva.fva_step(h, d_buf, tau, d_out, B, stream)
+    barrier()
+    sampler = ClockSampler(gpu_index_for(local_rank))
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        fva.fva_step(h, d_buf, tau, d_out, B, stream)
+    ev1.record(stream)
+    barrier()
+    clocks = sampler.stop()
+    ms = max_over_ranks(ev0.elapsed_time(ev1))
+    steps_total = args.steps * world
+    value = steps_total / (ms / 1e3)
+    us_per_step = 1e3 * ms / args.steps
+
+    # ---- end to end: pinned host buffer in, emitted chunk out, every step
+    h_buf = torch.from_numpy(buf).pin_memory()
+    h_out = torch.empty((B, wl.chunk_tokens, wl.action_dim)).pin_memory()
+    e2e_steps = max(10, args.steps // 4)
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            d_buf.copy_(h_buf, non_blocking=True)
+            fva.fva_step(h, d_buf, tau, d_out, B, stream)
+            h_out.copy_(d_out, non_blocking=True)
+        barrier()
+        ev0.record(stream)
+        for _ in range(e2e_steps):
+            d_buf.copy_(h_buf, non_blocking=True)
+            fva.fva_step(h, d_buf, tau, d_out, B, stream)
+            h_out.copy_(d_out, non_blocking=True)
+        ev1.record(stream)
+    barrier()
+    e2e_ms = max_over_ranks(ev0.elapsed_time(ev1))
+    e2e_value = e2e_steps * world / (e2e_ms / 1e3)
+    h2d = buf.nbytes + tau.nbytes
+    d2h = h_out.numel() * 4
+
+    # ---- kernel-by-kernel profile (CUDA events between launches on `stream`)
+    per_kind = {}
+    launches_per_step = 0
+    for _ in range(args.profile_steps):
+        recs = fva.fva_step_profile(h, d_buf, tau, d_out, B, stream)
+        launches_per_step = len(recs)
+        for kind, _layer, us in recs:
+            t, n = per_kind.get(kind, (0.0, 0))
+            per_kind[kind] = (t + us, n + 1)
+    prof_total = sum(t for t, _ in per_kind.values())
+    costs = kernel_costs(wl, B)
+    bw = peaks["hbm_gbs"] * 1e9
+    tc = peaks["bf16_tflops"] * 1e12
+    dom = max(per_kind, key=lambda k: per_kind[k][0])
+    t_us, n = per_kind[dom]
+    avg_s = t_us / n * 1e-6
+    fl, by = costs[dom]
+    if fl / tc >= by / bw:
+        roof = {"bound": "tensor", "achieved": fl / avg_s / 1e12, "peak": peaks["bf16_tflops"],
+                "unit": "TFLOP/s"}
+    else:
+        roof = {"bound": "hbm", "achieved": by / avg_s / 1e9, "peak": peaks["hbm_gbs"],
+                "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof.update({"traffic": None, "kernel": dom, "launches_per_step": per_kind[dom][1] //
+                 max(1, args.profile_steps), "avg_launch_us": t_us / n,
+                 "share_of_profiled_step": t_us / prof_total, "peak_source": f"{peak_src} burst"})
+    shares = {k: round(v[0] / prof_total, 4) for k, v in sorted(per_kind.items(),
+                                                                key=lambda kv: -kv[1][0])}
+
+    flops, nbytes = step_costs(wl, B)
+    t_roof = max(flops / tc, nbytes / bw)
+    step_roof = {"flops": flops, "bytes": nbytes, "t_tensor_us": 1e6 * flops / tc,
+                 "t_hbm_us": 1e6 * nbytes / bw, "roofline_us": 1e6 * t_roof,
+                 "frac": 1e6 * t_roof / us_per_step,
+                 "bound": "tensor" if flops / tc >= nbytes / bw else "hbm",
+                 "peaks": f"{peak_src}: {peaks['bf16_tflops']} TFLOP/s bf16 burst, "
+                          f"{peaks['hbm_gbs']} GB/s"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n_cpu, dt_cpu, cores = time_oracle(wl, w, pre, buf, tau, budget_s=args.cpu_budget,
+                                           max_steps=1000)
+        cpu = {"value": n_cpu / dt_cpu, "unit": "steps/s", "cores": cores, "kind": "oracle",
+               "sample": f"{n_cpu} full oracle steps of the same workload (fp64 NumPy)"}
+
+    dec.close()
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": args.gpus,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+                "us_per_step": us_per_step, "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": cfg_json,
+                "clocks": clocks,
+                "e2e": {"value": e2e_value, "unit": "steps/s", "h2d_bytes_per_step": h2d,
+                        "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+                "gpu_launches": launches_per_step * args.steps,
+                "roofline": roof, "step_roofline": step_roof, "kernel_shares": shares,
+                "cpu_baseline": cpu}
+        print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

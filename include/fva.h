@@ -1,0 +1,253 @@
+/*
+ * fva.h -- C ABI of the FlashVLA streaming action-decode library (libfva.so).
+ *
+ * FlashVLA (arXiv 2608.27384) decodes robot action chunks as a stream: a buffer of
+ * K action chunks, each H tokens of A action dimensions, holds the chunks at
+ * staggered noise levels tau_1 < ... < tau_K (§3.1, Eq. 2).  One forward pass of the
+ * flow-matching action expert, under a chunk-wise causal mask (§3.1), yields a
+ * velocity for every chunk; every chunk takes one Euler step toward its
+ * front neighbour's level (Eq. 1), the head chunk -- now clean -- is emitted as
+ * the executable action chunk, the others shift forward and fresh N(0, I) noise
+ * is pushed at the tail (§3.2, Algorithm 1, steady streaming).
+ *
+ * Everything on that path runs in this library's own CUDA kernels for sm_103a
+ * (GB300).  The library owns the weights, the cached prefix K/V and every
+ * workspace; the caller owns the streaming buffer, the output chunk and the
+ * CUDA stream.
+ *
+ * Conventions for every function:
+ *   - Return FVA_OK or an error code; no C++ exception crosses this boundary.
+ *   - Argument and state errors are detected on the host before any GPU work is
+ *     queued and leave every buffer untouched; fva_last_error() describes the
+ *     most recent error of the calling thread.
+ *   - Device pointers are plain CUDA device addresses on the device that was
+ *     current when fva_create ran; host pointers are ordinary host memory.
+ *   - Asynchronous CUDA faults surface as FVA_ERR_CUDA from a later call.
+ *   - A handle must not be used by two threads at once.
+ */
+#ifndef FVA_H_
+#define FVA_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define FVA_ABI_VERSION 1
+
+/* A CUDA stream (layout-compatible with cudaStream_t; NULL = legacy default stream). */
+typedef struct CUstream_st* fva_stream;
+
+typedef enum fva_status {
+  FVA_OK = 0,
+  FVA_ERR_INVALID_ARG = 1,  /* bad pointer, size, shape or value                      */
+  FVA_ERR_STATE = 2,        /* call out of order (e.g. step before weights / prefix) */
+  FVA_ERR_OOM = 3,          /* device or pinned-host allocation failed              */
+  FVA_ERR_CUDA = 4,         /* a CUDA runtime/driver call or a kernel failed        */
+  FVA_ERR_UNSUPPORTED = 5,  /* shape outside what the kernels of this dtype support */
+  FVA_ERR_TIMEOUT = 6       /* a kernel gave up a bounded wait (reported next call) */
+} fva_status;
+
+typedef enum fva_dtype {
+  FVA_FP32 = 0,  /* weights, activations and GEMMs in fp32 (CUDA-core path)            */
+  FVA_BF16 = 1   /* bf16 weights/activations, fp32 accumulate (tcgen05 tensor cores)   */
+} fva_dtype;
+
+/* fva_config.flags */
+#define FVA_FLAG_NO_GRAPH 1u  /* launch the step kernel by kernel instead of replaying a CUDA graph */
+
+/*
+ * Shape and numerics of the action expert and of the streaming buffer.
+ *
+ * The expert (App. A.4 of the paper: FiLM scale/shift/gate from the per-chunk
+ * timestep embedding; dimensions of a pi0.5-style expert) is: in-projection A->W;
+ * n_layers x [FiLM-modulated RMSNorm, MQA attention (n_q_heads query heads of
+ * head_dim, one KV head) with rotate-half RoPE, gated residual, FiLM-modulated
+ * RMSNorm, tanh-GELU gated MLP of mlp_dim, gated residual]; final FiLM-modulated
+ * RMSNorm; out-projection W->A.
+ *
+ * bf16 kernels support: head_dim == 256, n_q_heads in {1,2,4,8,16}, width and
+ * mlp_dim multiples of 128, action_dim <= 128.  fp32 kernels: any even head_dim
+ * <= 256, width a multiple of 4 (>= 8), action_dim <= 128.
+ */
+typedef struct fva_config {
+  int32_t abi_version;   /* must be FVA_ABI_VERSION                                  */
+  int32_t dtype;         /* fva_dtype                                                */
+  int32_t n_layers;      /* L                                                        */
+  int32_t width;         /* W, residual width                                        */
+  int32_t n_q_heads;     /* nq                                                       */
+  int32_t n_kv_heads;    /* must be 1 (multi-query attention)                        */
+  int32_t head_dim;      /* dh                                                       */
+  int32_t mlp_dim;       /* F                                                        */
+  int32_t action_dim;    /* A                                                        */
+  int32_t n_chunks;      /* K, buffer length (the paper's N)                         */
+  int32_t chunk_tokens;  /* H, tokens per chunk (the paper's chunk size C)           */
+  int32_t max_batch;     /* largest batch (independent requests) passed to fva_step */
+  int32_t max_prefix;    /* largest prefix length passed to fva_set_prefix_kv       */
+  uint32_t flags;        /* FVA_FLAG_*                                               */
+  float rms_eps;         /* RMSNorm epsilon (> 0)                                    */
+  float rope_theta;      /* RoPE base; 0 disables RoPE                               */
+  float t_min_period;    /* shortest period of the sinusoidal timestep embedding     */
+  float t_max_period;    /* longest period                                           */
+  uint64_t noise_seed;   /* Philox key of the tail noise drawn by fva_step           */
+} fva_config;
+
+typedef struct fva_handle fva_handle;
+
+/*
+ * Create a decoder on the current CUDA device: validates cfg, allocates every
+ * device buffer for max_batch requests (weights, prefix/action K/V workspace,
+ * activations, scratch) and zero-fills them.  *out receives the handle.
+ * Errors: INVALID_ARG (bad field), UNSUPPORTED (shape outside the dtype's
+ * kernels), OOM, CUDA.  Nothing is allocated when an error is returned.
+ */
+fva_status fva_create(const fva_config* cfg, fva_handle** out);
+
+/* Release every resource of h (NULL is a no-op).  Synchronises the device first. */
+void fva_destroy(fva_handle* h);
+
+/* Number of tensors fva_load_weights expects for cfg (0 if cfg is invalid). */
+int32_t fva_num_weights(const fva_config* cfg);
+
+/*
+ * Shape [rows, cols] (row-major, cols contiguous; vectors have rows == 1) of
+ * tensor `index` in the fva_load_weights order:
+ *   0 w_in [W, A]      1 b_in [W]      2 w_t1 [W, W]   3 b_t1 [W]
+ *   4 w_t2 [W, W]      5 b_t2 [W]
+ *   then for each layer l (base 6 + 11 l):
+ *     +0 w_mod1 [3W, W]  +1 b_mod1 [3W]   (scale | shift | gate, before attention)
+ *     +2 w_mod2 [3W, W]  +3 b_mod2 [3W]   (scale | shift | gate, before the MLP)
+ *     +4 w_q [nq dh, W]  +5 w_k [dh, W]   +6 w_v [dh, W]   +7 w_o [W, nq dh]
+ *     +8 w_gate [F, W]   +9 w_up [F, W]   +10 w_down [W, F]
+ *   then w_modf [2W, W], b_modf [2W] (scale | shift of the final norm),
+ *   w_out [A, W], b_out [A].
+ * Every matrix maps its input (cols) to its output (rows): y = x M^T + b.
+ */
+fva_status fva_weight_shape(const fva_config* cfg, int32_t index, int64_t* rows, int64_t* cols);
+
+/*
+ * Copy all weights into the library (the caller's arrays are not retained).
+ * tensors[i] points to tensor i above, element type = cfg.dtype (fp32, or bf16
+ * as raw uint16 bit patterns); on_device != 0 means device pointers, else host.
+ * May be called again to replace the weights.  Synchronous.
+ * Errors: INVALID_ARG (n_tensors != fva_num_weights, NULL entry), CUDA.
+ */
+fva_status fva_load_weights(fva_handle* h, const void* const* tensors, int32_t n_tensors,
+                            int32_t on_device);
+
+/*
+ * Install the cached VLM prefix keys/values of one observation for `request`
+ * (§3.1: every action token attends to the observation's prefix K/V).
+ * layer >= 0: k and v are [len, head_dim] for that layer; layer == -1: k and v
+ * are [n_layers, len, head_dim] for all layers.  Element type = cfg.dtype.  K is
+ * taken as already rotated by RoPE at positions 0..len-1; action token t of the
+ * request then sits at position len + t.  on_device selects device vs host
+ * pointers.  Copies are queued on `stream`; the caller's arrays may be reused
+ * once the stream reaches this point.  0 <= len <= max_prefix.  Every layer of a
+ * request must have the same len before fva_step uses that request.
+ */
+fva_status fva_set_prefix_kv(fva_handle* h, int32_t request, int32_t layer, const void* k,
+                             const void* v, int32_t len, int32_t on_device, fva_stream stream);
+
+/*
+ * One steady-streaming step (§3.2, Algorithm 1; Eq. 1 and 2) for `batch`
+ * independent requests, queued on `stream`; returns without waiting.
+ *   buffer       device fp32 [batch, K, H, A], slot 0 = cleanest chunk; updated in
+ *                place to [x'_2, ..., x'_K, z] where x'_k = x_k + dt_k v_k.
+ *   noise_levels host fp32 [batch, K]: tau_1 < ... < tau_K, each in (0, 1], per
+ *                request (read before the call returns).  dt_k = tau_{k-1} - tau_k
+ *                with tau_0 = 0, computed in fp32.
+ *   out_chunk    device fp32 [batch, H, A]: the emitted clean chunk x'_1.
+ *   batch        1 .. max_batch.
+ * The tail chunk z is drawn from Philox4x32-10 (key noise_seed, counter =
+ * (element/4, request, step index)) with Box-Muller; the step index starts at 0 and
+ * increases by one per call.  No allocation and no host synchronisation happen
+ * inside (except waiting for the parameter ring slot used `FVA_PARAM_RING` calls
+ * earlier).  Errors: INVALID_ARG (NULL, batch, non-increasing or out-of-range
+ * tau), STATE (no weights, a request without a complete prefix), TIMEOUT / CUDA
+ * (an earlier step failed on the GPU).
+ */
+fva_status fva_step(fva_handle* h, float* buffer, const float* noise_levels, float* out_chunk,
+                    int32_t batch, fva_stream stream);
+
+#define FVA_PARAM_RING 8
+
+/* Extra inputs / outputs of fva_step_ex (zero-initialise; every field optional). */
+typedef struct fva_step_opts {
+  const float* fresh_noise;  /* device fp32 [batch, H, A]: tail chunk to push instead of Philox */
+  float* velocity_out;       /* device fp32 [batch, K, H, A]: receives v                        */
+  int32_t trace_layer;       /* >= 0: write that layer's intermediates to trace_out            */
+  int32_t reserved;
+  float* trace_out;          /* device fp32, fva_trace_floats(h, batch) floats; see below      */
+} fva_step_opts;
+
+/*
+ * fva_step with options.  With trace_layer >= 0 the step runs kernel by kernel
+ * (no graph) and, for M = batch*K*H rows, writes fp32 copies of that layer's
+ * tensors to trace_out back to back in this order:
+ *   h_in [M, W], y1 [M, W], q [M, nq dh] (after RoPE), k [M, dh] (after RoPE),
+ *   v [M, dh], attn [M, nq dh], h_mid [M, W], y2 [M, W], mlp [M, F], h_out [M, W],
+ *   cond [batch*K, W] (per-chunk timestep condition).
+ */
+fva_status fva_step_ex(fva_handle* h, float* buffer, const float* noise_levels, float* out_chunk,
+                       int32_t batch, const fva_step_opts* opts, fva_stream stream);
+
+/* Floats needed by trace_out for `batch` (see fva_step_ex). */
+int64_t fva_trace_floats(const fva_handle* h, int32_t batch);
+
+/* Step index used for the next call's tail noise (checkpoint / resume of a stream). */
+fva_status fva_set_step_index(fva_handle* h, uint64_t step);
+fva_status fva_get_step_index(const fva_handle* h, uint64_t* step);
+
+/*
+ * The chunk-causal mask as the attention kernel applies it (§3.1): for each
+ * request r < batch and action token t < K*H, key_limit[r*K*H + t] receives the
+ * number of leading keys of [prefix_r ; action tokens of r] that the token
+ * attends to, P_r + (floor(t/H) + 1) H.  key_limit is a device int32 array.
+ */
+fva_status fva_mask_table(fva_handle* h, int32_t batch, int32_t* key_limit, fva_stream stream);
+
+/* Kernels of one step, as reported by fva_step_profile. */
+typedef enum fva_kernel_kind {
+  FVA_K_TIMESTEP_EMBED = 0,  /* sinusoidal embedding of every chunk's tau             */
+  FVA_K_TIME_MLP = 1,        /* one of the two SiLU linear layers of the condition   */
+  FVA_K_FILM = 2,            /* FiLM projections of every layer (one GEMM)           */
+  FVA_K_EMBED_NORM = 3,      /* action in-projection + layer-0 FiLM RMSNorm          */
+  FVA_K_QKV = 4,             /* packed QKV projection + RoPE + KV append             */
+  FVA_K_ATTENTION = 5,       /* chunk-causal MQA over prefix + action keys           */
+  FVA_K_OUT_PROJ = 6,        /* attention output projection (split-K partials)       */
+  FVA_K_RESID_NORM = 7,      /* split-K reduction + gated residual + FiLM RMSNorm    */
+  FVA_K_GATE_UP = 8,         /* packed gate/up projection + tanh-GELU gating         */
+  FVA_K_DOWN = 9,            /* MLP down projection (split-K partials)               */
+  FVA_K_FINAL = 10,          /* final norm + out-projection + Euler + emit + roll    */
+  FVA_K_COUNT = 11
+} fva_kernel_kind;
+
+typedef struct fva_kernel_time {
+  int32_t kind;        /* fva_kernel_kind                                    */
+  int32_t layer;       /* expert layer, or -1                                */
+  float microseconds;  /* CUDA-event time from this launch to the next one   */
+} fva_kernel_time;
+
+/*
+ * One step exactly like fva_step (same kernels, same results, advances the step
+ * index) but launched kernel by kernel with a CUDA event recorded before every
+ * launch and after the last; waits for the stream, then writes one record per
+ * launch, in launch order, to records[0 .. *n_records).  Each duration spans
+ * from the launch's own event to the next event on the stream, i.e. the kernel
+ * plus the launch gap after it.  Errors: as fva_step, plus INVALID_ARG when
+ * max_records is smaller than the number of launches.
+ */
+fva_status fva_step_profile(fva_handle* h, float* buffer, const float* noise_levels,
+                            float* out_chunk, int32_t batch, fva_kernel_time* records,
+                            int32_t max_records, int32_t* n_records, fva_stream stream);
+
+/* Description of the calling thread's most recent error ("" if none). */
+const char* fva_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FVA_H_ */

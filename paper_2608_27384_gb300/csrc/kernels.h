@@ -1,0 +1,149 @@
+// Internal interface between the host library (fva_api.cu) and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace fva {
+
+// Number of leading keys of [prefix ; action tokens] that action token t of a
+// request with prefix length P attends to under the chunk-wise causal mask
+// (own chunk bidirectional, earlier chunks fully, later chunks never).
+__host__ __device__ __forceinline__ int attn_key_limit(int P, int t, int H) {
+  return P + (t / H + 1) * H;
+}
+
+// Shapes of one step (all in elements).
+struct StepDims {
+  int B;       // active batch
+  int Bmax;    // allocated batch
+  int K, H, T; // chunks, tokens per chunk, K*H
+  int A, W, nq, dh, Dq, F, L;
+  int S_cap;   // KV rows per request and layer: max_prefix + T
+  int N_mod;   // FiLM outputs per chunk: L*6W + 2W
+  float eps;
+};
+
+// FiLM slice offsets inside one row of `mod` [B*K, N_mod].
+__host__ __device__ __forceinline__ int mod_off(int l, int which, int W) {
+  // which: 0 s1, 1 b1, 2 g1, 3 s2, 4 b2, 5 g2
+  return l * 6 * W + which * W;
+}
+__host__ __device__ __forceinline__ int modf_off(int L, int which, int W) {
+  // which: 0 sF, 1 bF
+  return L * 6 * W + which * W;
+}
+
+// ---------------------------------------------------------------- rowwise.cu
+// act_bf16 selects the activation type (bf16 when true, else fp32).
+void launch_temb(const float* tau, int rows, int W, float tmin, float tmax, void* out,
+                 bool act_bf16, cudaStream_t s);
+
+void launch_embed_norm(const StepDims& d, const float* buffer, const float* w_in_t,
+                       const float* b_in, const float* mod, float* h, void* y, bool act_bf16,
+                       cudaStream_t s);
+
+// h += gate * sum_z part[z];  y = rmsnorm(h) * (1 + scale) + shift.
+void launch_resid_norm(const StepDims& d, float* h, const float* part, int n_parts,
+                       long long part_stride, const float* mod, int gate_off, int scale_off,
+                       int shift_off, void* y, bool act_bf16, cudaStream_t s);
+
+// Final residual, final norm, out-projection, Euler update, emit, roll, tail.
+void launch_final(const StepDims& d, float* h, const float* part, int n_parts,
+                  long long part_stride, const float* mod, const float* w_out,
+                  const float* b_out, const float* dt, float* buffer, float* out_chunk,
+                  float* vel_out, const float* fresh, unsigned long long seed,
+                  const unsigned long long* step_idx, cudaStream_t s);
+
+void launch_rope_table(float2* table, int n_pos, int dh, float theta, cudaStream_t s);
+
+void launch_to_f32(const void* src, bool src_bf16, float* dst, long long n, cudaStream_t s);
+
+// Gather action-token K or V of one layer into a dense [B*T, dh] fp32 array.
+void launch_gather_action_kv(const void* kv_layer, bool act_bf16, const int* prefix_len,
+                             int B, int T, int S_cap, int dh, float* dst, cudaStream_t s);
+
+void launch_mask_table(const int* prefix_len, int B, int T, int H, int* key_limit,
+                       cudaStream_t s);
+
+// Gather rows: dst[r] = src[perm[r]] for rows of `row_bytes` bytes.
+void launch_row_gather(const void* src, void* dst, const int* perm, int rows, int row_bytes,
+                       cudaStream_t s);
+
+// ---------------------------------------------------------------- tc_gemm.cu
+enum GemmMode {
+  GEMM_BIAS_F32 = 0,      // out f32 = acc + bias
+  GEMM_BIAS_SILU_BF16 = 1,// out bf16 = silu(acc + bias)
+  GEMM_PARTIAL_F32 = 2,   // out f32 [split] = acc (split-K partial plane)
+  GEMM_QKV_ROPE = 3,      // RoPE, q -> q buffer, k/v -> KV workspace (permuted weights)
+  GEMM_GEGLU = 4,         // out bf16 = gelu(gate) * up (interleaved weights)
+};
+
+struct GemmEpi {
+  void* out;
+  const float* bias;
+  int ldo;
+  long long split_stride;
+  // GEMM_QKV_ROPE
+  void* q;
+  void* kc;             // layer's [Bmax, S_cap, dh]
+  void* vc;
+  const int* prefix_len;
+  const float2* rope;   // [n_pos, dh/2] (cos, sin)
+  int T, S_cap, nq, dh;
+  int* err;
+};
+
+// Tile widths used for each GEMM of the step (the weight layouts depend on them).
+constexpr int kBnQKV = 128;
+constexpr int kBnGU = 256;
+constexpr int kBnResid = 128;
+constexpr int kBnTime = 64;
+constexpr int kBnFilm = 256;
+
+// Prepare kernel attributes (max dynamic shared memory); call once per device.
+cudaError_t tc_gemm_init();
+
+// C = A[M, K] * B[N, K]^T on tcgen05 with the given epilogue.
+// K must be a multiple of 64 and N of bn; M is any positive size.
+cudaError_t launch_tc_gemm(int bn, int mode, const CUtensorMap* a, const CUtensorMap* b,
+                           const GemmEpi& ep, int M, int N, int K, int splits,
+                           cudaStream_t s);
+
+// ---------------------------------------------------------------- tc_attention.cu
+struct AttnArgs {
+  const int* prefix_len;
+  void* out;            // bf16 [Bmax*T*nq, 256]
+  float* part_o;        // [B*tiles, max_splits, 128, 256]
+  float2* part_ml;      // [B*tiles, max_splits, 128]
+  int* counters;        // [Bmax*tiles], zero between launches
+  int T, H, nq, S_cap, tiles_per_req, max_splits;
+  int kv_row0;          // first KV row of this layer in the 2D view
+  float scale_log2;     // log2(e) / sqrt(dh)
+  int* err;
+};
+
+constexpr int kAttnKeysPerSplit = 256;
+constexpr int kAttnKeyBlock = 64;
+
+cudaError_t tc_attention_init();
+cudaError_t launch_tc_attention(const CUtensorMap* q, const CUtensorMap* k,
+                                const CUtensorMap* v, const AttnArgs& a, int B,
+                                cudaStream_t s);
+
+// ---------------------------------------------------------------- simt_f32.cu
+// C[M, N] = A[M, K] (lda) * B[N, K]^T, fp32 on CUDA cores.
+void launch_f32_gemm(const float* A, int lda, const float* B, float* C, int ldc, int M, int N,
+                     int K, cudaStream_t s);
+void launch_f32_bias_act(const float* C, const float* bias, float* out, int M, int N,
+                         bool silu, cudaStream_t s);
+void launch_f32_qkv_rope(const float* C, float* q, float* kc, float* vc,
+                         const int* prefix_len, const float2* rope, int M, int T, int S_cap,
+                         int nq, int dh, cudaStream_t s);
+void launch_f32_geglu(const float* C, float* out, int M, int F, cudaStream_t s);
+void launch_f32_attention(const float* q, const float* kc, const float* vc,
+                          const int* prefix_len, float* out, int B, int T, int H, int nq,
+                          int dh, int S_cap, int max_keys, cudaStream_t s);
+
+}  // namespace fva

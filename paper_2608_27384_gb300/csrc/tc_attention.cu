@@ -1,0 +1,307 @@
+// Chunk-wise causal multi-query attention on tcgen05 (head_dim 256, bf16).
+//
+// The paper's mask (§3.1): action token t of chunk c(t) = floor(t / H) attends to
+// every prefix key of its request and to the action keys of chunks <= c(t)
+// (bidirectional inside its own chunk).  In the concatenated key sequence
+// [prefix ; action tokens] that is the leading range [0, P + (c(t)+1) H).
+//
+// Work decomposition.  A query tile is 128 rows = 128/nq consecutive tokens x
+// all nq heads of one request: MQA heads share the single KV head, so one K/V
+// tile in shared memory serves every head.  The key range of a tile is cut into
+// splits of 256 keys (4 blocks of 64); key blocks past the tile's largest limit
+// are never loaded.  One CTA handles one (tile, split):
+//   warp 0      TMA: Q tile (64 KB, loaded once) then K blocks, then V blocks,
+//               through a 2-slot ring of 32 KB;
+//   warp 1      TMEM (512 columns: S in 0..255, O in 256..511); one lane issues
+//               S = Q K^T per key block (M=128, N=64, K=16 steps over dh), and,
+//               after the softmax, O = P V (M=128, N=256, MN-major V);
+//   warps 2..5  one thread per query row: exact row max over the split's visible
+//               keys, P = exp(S - max) written as bf16 into the swizzled A-operand
+//               layout in shared memory, row sum; then read O from TMEM.
+// A tile with one split writes O / l as bf16.  Otherwise each split writes its
+// (O, max, sum) to scratch and the last CTA of the tile (atomic ticket) merges
+// the splits in split order -- deterministic -- and writes bf16.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace fva {
+
+namespace {
+
+constexpr int kDH = 256;
+constexpr int kRows = 128;
+constexpr int kKB = kAttnKeyBlock;                    // 64 keys per block
+constexpr int kBlocksPerSplit = kAttnKeysPerSplit / kKB;  // 4
+constexpr int kQBytes = kRows * kDH * 2;              // 64 KB
+constexpr int kPBytes = kRows * kAttnKeysPerSplit * 2;  // 64 KB
+constexpr int kKVBytes = kKB * kDH * 2;               // 32 KB per K or V block
+constexpr int kSlots = 2;
+constexpr int kSmem = kQBytes + kPBytes + kSlots * kKVBytes + 1024 + 256;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 512;
+
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
+  const int tile = blockIdx.x, split = blockIdx.y, r = blockIdx.z;
+  const int tok_per_tile = kRows / a.nq;
+  const int t0 = tile * tok_per_tile;
+  const int t_last = min(a.T, t0 + tok_per_tile) - 1;
+  const int P = __ldg(a.prefix_len + r);
+  const int limit_max = attn_key_limit(P, t_last, a.H);
+  const int nkb_tile = (limit_max + kKB - 1) / kKB;
+  const int nsplit = (nkb_tile + kBlocksPerSplit - 1) / kBlocksPerSplit;
+  if (split >= nsplit) return;  // uniform over the CTA, before any barrier / TMEM use
+  const int kb0 = split * kBlocksPerSplit;
+  const int nblk = min(kBlocksPerSplit, nkb_tile - kb0);
+
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sQ = smem;                       // 4 slabs [128 rows x 128 B]
+  uint8_t* sP = smem + kQBytes;             // 4 slabs [128 rows x 128 B]
+  uint8_t* sKV = sP + kPBytes;              // 2 slots x 4 slabs [64 rows x 128 B]
+  uint64_t* bars = (uint64_t*)(sKV + kSlots * kKVBytes);
+  uint64_t* q_full = bars + 0;
+  uint64_t* kv_full = bars + 1;   // [2]
+  uint64_t* kv_empty = bars + 3;  // [2]
+  uint64_t* s_full = bars + 5;
+  uint64_t* p_full = bars + 6;
+  uint64_t* o_full = bars + 7;
+  uint32_t* tmem_slot = (uint32_t*)(bars + 8);
+  int* last_flag = (int*)(bars + 9);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < kSlots; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    mbar_init(s_full, 1);
+    mbar_init(p_full, kRows);
+    mbar_init(o_full, 1);
+    fence_barrier_init();
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmV);
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t tS = tmem, tO = tmem + 256;
+
+  const int qrow0 = (r * a.T + t0) * a.nq;
+  const int krow0 = a.kv_row0 + r * a.S_cap + kb0 * kKB;
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer
+    mbar_arrive_expect_tx(q_full, kQBytes);
+    for (int j = 0; j < 4; ++j) tma_load_2d(sQ + j * (kRows * 128), &tmQ, j * 64, qrow0, q_full);
+    for (int it = 0; it < 2 * nblk; ++it) {
+      const int s = it & 1;
+      const uint32_t ph = (uint32_t)(it >> 1) & 1u;
+      if (!mbar_wait(&kv_empty[s], ph ^ 1u, a.err, KERR_WAIT_MMA)) break;
+      const bool is_k = it < nblk;
+      const int row = krow0 + (is_k ? it : it - nblk) * kKB;
+      uint8_t* dst = sKV + s * kKVBytes;
+      mbar_arrive_expect_tx(&kv_full[s], kKVBytes);
+      for (int j = 0; j < 4; ++j)
+        tma_load_2d(dst + j * (kKB * 128), is_k ? &tmK : &tmV, j * 64, row, &kv_full[s]);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer
+    constexpr uint32_t idesc_s = umma_idesc_bf16(kRows, kKB, false);
+    constexpr uint32_t idesc_o = umma_idesc_bf16(kRows, kDH, true);
+    bool good = mbar_wait(q_full, 0, a.err, KERR_WAIT_TMA);
+    tc_fence_after();
+    const uint32_t q_base = smem_u32(sQ), p_base = smem_u32(sP), kv_base = smem_u32(sKV);
+    for (int it = 0; good && it < nblk; ++it) {
+      const int s = it & 1;
+      if (!mbar_wait(&kv_full[s], (uint32_t)(it >> 1) & 1u, a.err, KERR_WAIT_TMA)) {
+        good = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t kb = kv_base + s * kKVBytes;
+#pragma unroll
+      for (int ks = 0; ks < kDH / 16; ++ks) {
+        const uint32_t off = (ks & 3) * 32;  // 16 bf16 along K inside the 128-byte row
+        const uint64_t ad = umma_desc_sw128(q_base + (ks >> 2) * (kRows * 128) + off, 16, 1024);
+        const uint64_t bd = umma_desc_sw128(kb + (ks >> 2) * (kKB * 128) + off, 16, 1024);
+        umma_bf16(tS + it * kKB, ad, bd, idesc_s, ks > 0 ? 1u : 0u);
+      }
+      umma_commit(&kv_empty[s]);
+    }
+    if (good) umma_commit(s_full);
+    if (good) good = mbar_wait(p_full, 0, a.err, KERR_WAIT_SYNC);
+    tc_fence_after();
+    for (int j = 0; good && j < nblk; ++j) {
+      const int it = nblk + j, s = it & 1;
+      if (!mbar_wait(&kv_full[s], (uint32_t)(it >> 1) & 1u, a.err, KERR_WAIT_TMA)) {
+        good = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t vb = kv_base + s * kKVBytes;
+#pragma unroll
+      for (int ks = 0; ks < kKB / 16; ++ks) {
+        const uint64_t ad = umma_desc_sw128(p_base + j * (kRows * 128) + ks * 32, 16, 1024);
+        // V block [64 keys][256 dh] as 4 slabs of 64 dh: MN-major B operand.
+        const uint64_t bd = umma_desc_sw128(vb + ks * 16 * 128, kKB * 128, 1024);
+        umma_bf16(tO, ad, bd, idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
+      }
+      umma_commit(&kv_empty[s]);
+    }
+    if (good) umma_commit(o_full);
+  } else if (warp >= 2) {
+    // ---------------- softmax + epilogue, one query row per thread
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    const int t = t0 + row / a.nq;
+    const bool valid = t < a.T;
+    const int limit = valid ? attn_key_limit(P, t, a.H) : 0;
+    const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+    bool good = __all_sync(0xffffffffu, mbar_wait(s_full, 0, a.err, KERR_WAIT_MMA));
+    tc_fence_after();
+    float mx = -INFINITY, l = 0.f;
+    if (good) {
+      for (int j = 0; j < nblk; ++j) {
+        for (int hh = 0; hh < 2; ++hh) {
+          float v[32];
+          tmem_ld32(tS + lane_off + j * kKB + hh * 32, v);
+          const int key0 = (kb0 + j) * kKB + hh * 32;
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (key0 + i < limit) mx = fmaxf(mx, v[i]);
+        }
+      }
+      const float mscaled = mx * a.scale_log2;
+      for (int j = 0; j < nblk; ++j) {
+        uint8_t* prow = sP + j * (kRows * 128) + row * 128;
+        for (int hh = 0; hh < 2; ++hh) {
+          float v[32];
+          tmem_ld32(tS + lane_off + j * kKB + hh * 32, v);
+          const int key0 = (kb0 + j) * kKB + hh * 32;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float p = (key0 + i < limit) ? exp2f(fmaf(v[i], a.scale_log2, -mscaled)) : 0.f;
+            const float pr = __bfloat162float(__float2bfloat16_rn(p));
+            l += pr;
+            v[i] = pr;
+          }
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const int chunk = hh * 4 + c;                       // 16-byte chunk in the row
+            const int phys = chunk ^ (row & 7);                 // 128-byte swizzle
+            *reinterpret_cast<uint4*>(prow + phys * 16) = pack_bf16x8(&v[c * 8]);
+          }
+        }
+      }
+    }
+    fence_proxy_async_smem();
+    mbar_arrive(p_full);
+    if (good) good = __all_sync(0xffffffffu, mbar_wait(o_full, 0, a.err, KERR_WAIT_MMA));
+    tc_fence_after();
+    const int n_tiles_req = a.tiles_per_req;
+    const int gtile = r * n_tiles_req + tile;
+    const int grow = qrow0 + row;  // global q row = (r*T + t) * nq + head
+    if (good) {
+      if (nsplit == 1) {
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        for (int c = 0; c < kDH; c += 32) {
+          float v[32];
+          tmem_ld32(tO + lane_off + c, v);
+          if (!valid) continue;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] *= inv;
+          bf16* dst = (bf16*)a.out + (size_t)grow * kDH + c;
+#pragma unroll
+          for (int i = 0; i < 32; i += 8) *reinterpret_cast<uint4*>(dst + i) = pack_bf16x8(&v[i]);
+        }
+      } else {
+        float* po = a.part_o + (((size_t)gtile * a.max_splits + split) * kRows + row) * kDH;
+        for (int c = 0; c < kDH; c += 32) {
+          float v[32];
+          tmem_ld32(tO + lane_off + c, v);
+#pragma unroll
+          for (int i = 0; i < 32; i += 4)
+            __stcg(reinterpret_cast<float4*>(po + c + i), make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]));
+        }
+        __stcg(a.part_ml + ((size_t)gtile * a.max_splits + split) * kRows + row,
+               make_float2(mx, l));
+      }
+    }
+    if (nsplit > 1) {
+      // last-arriving split of this tile merges all splits in split order
+      __threadfence();
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (warp == 2 && lane == 0) {
+        const int ticket = atomicAdd(a.counters + gtile, 1);
+        *last_flag = (ticket == nsplit - 1) ? 1 : 0;
+        if (ticket == nsplit - 1) a.counters[gtile] = 0;  // ready for the next launch
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (*last_flag) {
+        __threadfence();
+        if (valid) {
+          float m_all = -INFINITY;
+          for (int s = 0; s < nsplit; ++s) {
+            const float2 ml = __ldcg(a.part_ml + ((size_t)gtile * a.max_splits + s) * kRows + row);
+            if (ml.y > 0.f) m_all = fmaxf(m_all, ml.x);
+          }
+          float wsum = 0.f, wts[32];
+          const int ns = min(nsplit, 32);
+          for (int s = 0; s < ns; ++s) {
+            const float2 ml = __ldcg(a.part_ml + ((size_t)gtile * a.max_splits + s) * kRows + row);
+            const float w = ml.y > 0.f ? exp2f((ml.x - m_all) * a.scale_log2) : 0.f;
+            wts[s] = w;
+            wsum += w * ml.y;
+          }
+          const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+          for (int c = 0; c < kDH; c += 8) {
+            float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+            for (int s = 0; s < ns; ++s) {
+              const float* po =
+                  a.part_o + (((size_t)gtile * a.max_splits + s) * kRows + row) * kDH + c;
+              const float4 x0 = __ldcg(reinterpret_cast<const float4*>(po));
+              const float4 x1 = __ldcg(reinterpret_cast<const float4*>(po + 4));
+              const float w = wts[s];
+              acc[0] = fmaf(w, x0.x, acc[0]); acc[1] = fmaf(w, x0.y, acc[1]);
+              acc[2] = fmaf(w, x0.z, acc[2]); acc[3] = fmaf(w, x0.w, acc[3]);
+              acc[4] = fmaf(w, x1.x, acc[4]); acc[5] = fmaf(w, x1.y, acc[5]);
+              acc[6] = fmaf(w, x1.z, acc[6]); acc[7] = fmaf(w, x1.w, acc[7]);
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) acc[i] *= inv;
+            *reinterpret_cast<uint4*>((bf16*)a.out + (size_t)grow * kDH + c) = pack_bf16x8(acc);
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace
+
+cudaError_t tc_attention_init() {
+  return cudaFuncSetAttribute(tc_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+}
+
+cudaError_t launch_tc_attention(const CUtensorMap* q, const CUtensorMap* k,
+                                const CUtensorMap* v, const AttnArgs& a, int B,
+                                cudaStream_t s) {
+  if (a.max_splits > 32) return cudaErrorInvalidValue;  // merge keeps <= 32 weights in registers
+  dim3 grid(a.tiles_per_req, a.max_splits, B);
+  tc_attn_kernel<<<grid, kThreads, kSmem, s>>>(*q, *k, *v, a);
+  return cudaGetLastError();
+}
+
+}  // namespace fva
