@@ -148,7 +148,6 @@ struct fva_handle {
   float* fresh = nullptr;
   float* att_part_o = nullptr;
   float2* att_part_ml = nullptr;
-  int* att_counters = nullptr;
   int* err_dev = nullptr;
   CUtensorMap m_temb, m_t1, m_cond, m_y, m_attn, m_mlp, m_q, m_k, m_v;
   // per-step parameters: [tau BKmax | dt BKmax | step u64]
@@ -368,8 +367,7 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
     h->attn_max_splits = (h->S_cap + kAttnKeysPerSplit - 1) / kAttnKeysPerSplit;
     const size_t tiles = (size_t)h->Bmax * h->tiles_per_req;
     if ((st = dalloc(h, &h->att_part_o, tiles * h->attn_max_splits * 128 * 256)) ||
-        (st = dalloc(h, &h->att_part_ml, tiles * h->attn_max_splits * 128)) ||
-        (st = dalloc(h, &h->att_counters, tiles)))
+        (st = dalloc(h, &h->att_part_ml, tiles * h->attn_max_splits * 128)))
       return st;
   }
   h->params_floats = 2 * h->BKmax + 2;
@@ -827,7 +825,6 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       aa.out = h->attn;
       aa.part_o = h->att_part_o;
       aa.part_ml = h->att_part_ml;
-      aa.counters = h->att_counters;
       aa.T = h->T;
       aa.H = h->H;
       aa.nq = h->nq;

@@ -67,9 +67,6 @@ void launch_gather_action_kv(const void* kv_layer, bool act_bf16, const int* pre
 void launch_mask_table(const int* prefix_len, int B, int T, int H, int* key_limit,
                        cudaStream_t s);
 
-// Gather rows: dst[r] = src[perm[r]] for rows of `row_bytes` bytes.
-void launch_row_gather(const void* src, void* dst, const int* perm, int rows, int row_bytes,
-                       cudaStream_t s);
 
 // ---------------------------------------------------------------- tc_gemm.cu
 enum GemmMode {
@@ -117,7 +114,6 @@ struct AttnArgs {
   void* out;            // bf16 [Bmax*T*nq, 256]
   float* part_o;        // [B*tiles, max_splits, 128, 256]
   float2* part_ml;      // [B*tiles, max_splits, 128]
-  int* counters;        // [Bmax*tiles], zero between launches
   int T, H, nq, S_cap, tiles_per_req, max_splits;
   int kv_row0;          // first KV row of this layer in the 2D view
   float scale_log2;     // log2(e) / sqrt(dh)
@@ -128,6 +124,7 @@ constexpr int kAttnKeysPerSplit = 256;
 constexpr int kAttnKeyBlock = 64;
 
 cudaError_t tc_attention_init();
+// Attention kernel, then (when a tile can have several key splits) the merge kernel.
 cudaError_t launch_tc_attention(const CUtensorMap* q, const CUtensorMap* k,
                                 const CUtensorMap* v, const AttnArgs& a, int B,
                                 cudaStream_t s);

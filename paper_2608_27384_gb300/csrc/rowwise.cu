@@ -17,6 +17,8 @@ __global__ void temb_kernel(const float* __restrict__ tau, int W, double tmin, d
                             Act* __restrict__ out) {
   const int row = blockIdx.x;
   const int half = W / 2;
+  pdl_trigger();
+  pdl_wait();
   const double t = (double)tau[row];
   for (int j = threadIdx.x; j < half; j += blockDim.x) {
     const double period = tmin * pow(tmax / tmin, (double)j / (double)(half - 1));
@@ -32,13 +34,15 @@ void launch_temb(const float* tau, int rows, int W, float tmin, float tmax, void
                  bool act_bf16, cudaStream_t s) {
   if (rows <= 0) return;
   if (act_bf16)
-    temb_kernel<bf16><<<rows, 256, 0, s>>>(tau, W, tmin, tmax, (bf16*)out);
+    launch_pdl(temb_kernel<bf16>, dim3(rows), dim3(256), 0, s, tau, W, (double)tmin,
+               (double)tmax, (bf16*)out);
   else
-    temb_kernel<float><<<rows, 256, 0, s>>>(tau, W, tmin, tmax, (float*)out);
+    launch_pdl(temb_kernel<float>, dim3(rows), dim3(256), 0, s, tau, W, (double)tmin,
+               (double)tmax, (float*)out);
 }
 
 // ----------------------------------------------------------------------------
-// helpers for one row held by one warp (W a multiple of 4)
+// row helpers (W a multiple of 4)
 // ----------------------------------------------------------------------------
 template <typename Act>
 __device__ __forceinline__ void store4(Act* dst, float a, float b, float c, float d);
@@ -55,14 +59,27 @@ __device__ __forceinline__ void store4<bf16>(bf16* dst, float a, float b, float 
   *reinterpret_cast<uint2*>(dst) = u;
 }
 
-// y = h * rsqrt(mean(h^2) + eps) * (1 + scale) + shift  for a row already in h.
+// Sum over the CTA (blockDim.x a multiple of 32, at most 1024); every thread gets it.
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  v = warp_sum(v);
+  __syncthreads();  // red may still be read by a previous call
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float t = 0.f;
+  for (int w = 0; w < nw; ++w) t += red[w];
+  return t;
+}
+
+// y = h * rsqrt(mean(h^2) + eps) * (1 + scale) + shift for a row already in h
+// (each thread re-reads the columns it wrote itself).
 template <typename Act>
 __device__ __forceinline__ void modulated_norm_row(const float* __restrict__ hrow, float ss, int W,
                                                    float eps, const float* __restrict__ scale,
                                                    const float* __restrict__ shift,
-                                                   Act* __restrict__ yrow, int lane) {
+                                                   Act* __restrict__ yrow) {
   const float r = rsqrtf(ss / (float)W + eps);
-  for (int c = lane * 4; c < W; c += 128) {
+  for (int c = threadIdx.x * 4; c < W; c += blockDim.x * 4) {
     const float4 hv = *reinterpret_cast<const float4*>(hrow + c);
     const float4 sc = *reinterpret_cast<const float4*>(scale + c);
     const float4 sh = *reinterpret_cast<const float4*>(shift + c);
@@ -71,26 +88,36 @@ __device__ __forceinline__ void modulated_norm_row(const float* __restrict__ hro
   }
 }
 
+inline int row_threads(int W) {
+  int t = W / 4;
+  t = t < 32 ? 32 : (t > 256 ? 256 : t);
+  return (t + 31) & ~31;
+}
+
 // ----------------------------------------------------------------------------
 // action in-projection h = x W_in^T + b_in, then layer 0's FiLM RMSNorm.
-// One warp per token row; w_in_t is W_in transposed, [A, W] fp32.
+// One CTA per token row; w_in_t is W_in transposed, [A, W] fp32.
 // ----------------------------------------------------------------------------
 template <typename Act>
 __global__ void embed_norm_kernel(StepDims d, const float* __restrict__ buffer,
                                   const float* __restrict__ w_in_t,
                                   const float* __restrict__ b_in, const float* __restrict__ mod,
                                   float* __restrict__ h, Act* __restrict__ y) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m = blockIdx.x * (blockDim.x >> 5) + warp;
-  if (m >= d.B * d.T) return;
+  __shared__ float xs[128];
+  __shared__ float red[32];
+  const int m = blockIdx.x;
   const int r = m / d.T, t = m % d.T, c = t / d.H;
+  pdl_trigger();
+  pdl_wait();
   const float* x = buffer + (size_t)m * d.A;  // buffer [B, K, H, A] = rows of A
+  for (int a = threadIdx.x; a < d.A; a += blockDim.x) xs[a] = x[a];
+  __syncthreads();
   float* hrow = h + (size_t)m * d.W;
   float ss = 0.f;
-  for (int col = lane * 4; col < d.W; col += 128) {
+  for (int col = threadIdx.x * 4; col < d.W; col += blockDim.x * 4) {
     float4 acc = *reinterpret_cast<const float4*>(b_in + col);
     for (int a = 0; a < d.A; ++a) {
-      const float xa = x[a];
+      const float xa = xs[a];
       const float4 w = *reinterpret_cast<const float4*>(w_in_t + (size_t)a * d.W + col);
       acc.x = fmaf(xa, w.x, acc.x);
       acc.y = fmaf(xa, w.y, acc.y);
@@ -100,26 +127,28 @@ __global__ void embed_norm_kernel(StepDims d, const float* __restrict__ buffer,
     *reinterpret_cast<float4*>(hrow + col) = acc;
     ss += acc.x * acc.x + acc.y * acc.y + acc.z * acc.z + acc.w * acc.w;
   }
-  ss = warp_sum(ss);
+  ss = block_sum(ss, red);
   const float* mrow = mod + (size_t)(r * d.K + c) * d.N_mod;
   modulated_norm_row<Act>(hrow, ss, d.W, d.eps, mrow + mod_off(0, 0, d.W),
-                          mrow + mod_off(0, 1, d.W), y + (size_t)m * d.W, lane);
+                          mrow + mod_off(0, 1, d.W), y + (size_t)m * d.W);
 }
 
 void launch_embed_norm(const StepDims& d, const float* buffer, const float* w_in_t,
                        const float* b_in, const float* mod, float* h, void* y, bool act_bf16,
                        cudaStream_t s) {
-  const int rows = d.B * d.T, wpb = 8;
-  dim3 grid((rows + wpb - 1) / wpb);
+  const int rows = d.B * d.T;
+  if (rows <= 0) return;
   if (act_bf16)
-    embed_norm_kernel<bf16><<<grid, 32 * wpb, 0, s>>>(d, buffer, w_in_t, b_in, mod, h, (bf16*)y);
+    launch_pdl(embed_norm_kernel<bf16>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, buffer,
+               w_in_t, b_in, mod, h, (bf16*)y);
   else
-    embed_norm_kernel<float><<<grid, 32 * wpb, 0, s>>>(d, buffer, w_in_t, b_in, mod, h, (float*)y);
+    launch_pdl(embed_norm_kernel<float>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, buffer,
+               w_in_t, b_in, mod, h, (float*)y);
 }
 
 // ----------------------------------------------------------------------------
 // h += gate_c * sum_z part[z]  (split-K partials reduced in fixed order z = 0..),
-// then y = FiLM RMSNorm(h) with the next norm's (scale, shift).
+// then y = FiLM RMSNorm(h) with the next norm's (scale, shift).  One CTA per row.
 // ----------------------------------------------------------------------------
 template <typename Act>
 __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
@@ -127,14 +156,15 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
                                   long long part_stride, const float* __restrict__ mod,
                                   int gate_off, int scale_off, int shift_off,
                                   Act* __restrict__ y) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m = blockIdx.x * (blockDim.x >> 5) + warp;
-  if (m >= d.B * d.T) return;
+  __shared__ float red[32];
+  const int m = blockIdx.x;
   const int r = m / d.T, c = (m % d.T) / d.H;
+  pdl_trigger();
+  pdl_wait();
   const float* mrow = mod + (size_t)(r * d.K + c) * d.N_mod;
   float* hrow = h + (size_t)m * d.W;
   float ss = 0.f;
-  for (int col = lane * 4; col < d.W; col += 128) {
+  for (int col = threadIdx.x * 4; col < d.W; col += blockDim.x * 4) {
     float4 acc = __ldcg(reinterpret_cast<const float4*>(part + (size_t)m * d.W + col));
     for (int z = 1; z < n_parts; ++z) {
       const float4 p =
@@ -150,23 +180,22 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
     *reinterpret_cast<float4*>(hrow + col) = hv;
     ss += hv.x * hv.x + hv.y * hv.y + hv.z * hv.z + hv.w * hv.w;
   }
-  ss = warp_sum(ss);
-  if (y == nullptr) return;
+  ss = block_sum(ss, red);
   modulated_norm_row<Act>(hrow, ss, d.W, d.eps, mrow + scale_off, mrow + shift_off,
-                          y + (size_t)m * d.W, lane);
+                          y + (size_t)m * d.W);
 }
 
 void launch_resid_norm(const StepDims& d, float* h, const float* part, int n_parts,
                        long long part_stride, const float* mod, int gate_off, int scale_off,
                        int shift_off, void* y, bool act_bf16, cudaStream_t s) {
-  const int rows = d.B * d.T, wpb = 8;
-  dim3 grid((rows + wpb - 1) / wpb);
+  const int rows = d.B * d.T;
+  if (rows <= 0) return;
   if (act_bf16)
-    resid_norm_kernel<bf16><<<grid, 32 * wpb, 0, s>>>(d, h, part, n_parts, part_stride, mod,
-                                                      gate_off, scale_off, shift_off, (bf16*)y);
+    launch_pdl(resid_norm_kernel<bf16>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h, part,
+               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (bf16*)y);
   else
-    resid_norm_kernel<float><<<grid, 32 * wpb, 0, s>>>(d, h, part, n_parts, part_stride, mod,
-                                                       gate_off, scale_off, shift_off, (float*)y);
+    launch_pdl(resid_norm_kernel<float>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h, part,
+               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (float*)y);
 }
 
 // ----------------------------------------------------------------------------
@@ -222,6 +251,8 @@ __global__ void final_kernel(StepDims d, float* __restrict__ h, const float* __r
   const int j = blockIdx.x, r = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
   const int lgate = mod_off(d.L - 1, 5, d.W);
+  pdl_trigger();
+  pdl_wait();
   for (int k = warp; k < d.K; k += nw) {
     const int t = k * d.H + j;
     const size_t m = (size_t)r * d.T + t;
@@ -279,8 +310,7 @@ __global__ void final_kernel(StepDims d, float* __restrict__ h, const float* __r
   for (int a = threadIdx.x; a < d.A; a += blockDim.x) {
     float* col = buffer + ((size_t)r * d.K * d.H + j) * d.A + a;  // + k*H*A selects the slot
     const size_t slot = (size_t)d.H * d.A;
-    float nxt = __fadd_rn(col[0], __fmul_rn(dtr[0], vs[a]));
-    out_chunk[((size_t)r * d.H + j) * d.A + a] = nxt;
+    out_chunk[((size_t)r * d.H + j) * d.A + a] = __fadd_rn(col[0], __fmul_rn(dtr[0], vs[a]));
     if (vel_out) vel_out[((size_t)r * d.K * d.H + j) * d.A + a] = vs[a];
     for (int k = 1; k < d.K; ++k) {
       const float v = vs[k * d.A + a];
@@ -291,7 +321,6 @@ __global__ void final_kernel(StepDims d, float* __restrict__ h, const float* __r
     const int e = j * d.A + a;
     col[(size_t)(d.K - 1) * slot] =
         fresh ? fresh[(size_t)r * d.H * d.A + e] : tail_normal(seed, step, r, e);
-    (void)nxt;
   }
 }
 
@@ -302,8 +331,8 @@ void launch_final(const StepDims& d, float* h, const float* part, int n_parts,
                   const unsigned long long* step_idx, cudaStream_t s) {
   dim3 grid(d.H, d.B);
   const size_t smem = sizeof(float) * d.K * d.A;
-  final_kernel<<<grid, 256, smem, s>>>(d, h, part, n_parts, part_stride, mod, w_out, b_out, dt,
-                                       buffer, out_chunk, vel_out, fresh, seed, step_idx);
+  launch_pdl(final_kernel, grid, dim3(256), smem, s, d, h, part, n_parts, part_stride, mod,
+             w_out, b_out, dt, buffer, out_chunk, vel_out, fresh, seed, step_idx);
 }
 
 // ----------------------------------------------------------------------------
@@ -331,6 +360,7 @@ void launch_rope_table(float2* table, int n_pos, int dh, float theta, cudaStream
 }
 
 __global__ void to_f32_kernel(const void* src, bool src_bf16, float* dst, long long n) {
+  pdl_wait();
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n;
        i += (long long)gridDim.x * blockDim.x)
     dst[i] = src_bf16 ? __bfloat162float(((const bf16*)src)[i]) : ((const float*)src)[i];
@@ -344,6 +374,7 @@ __global__ void gather_action_kv_kernel(const void* kv, bool act_bf16,
                                         const int* __restrict__ prefix_len, int T, int S_cap,
                                         int dh, float* dst) {
   const int m = blockIdx.x, r = m / T, t = m % T;
+  pdl_wait();
   const size_t row = (size_t)r * S_cap + prefix_len[r] + t;
   for (int i = threadIdx.x; i < dh; i += blockDim.x)
     dst[(size_t)m * dh + i] = act_bf16 ? __bfloat162float(((const bf16*)kv)[row * dh + i])
@@ -359,6 +390,7 @@ void launch_gather_action_kv(const void* kv_layer, bool act_bf16, const int* pre
 __global__ void mask_table_kernel(const int* __restrict__ prefix_len, int B, int T, int H,
                                   int* key_limit) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  pdl_wait();
   if (i >= B * T) return;
   key_limit[i] = attn_key_limit(prefix_len[i / T], i % T, H);
 }
@@ -366,20 +398,6 @@ __global__ void mask_table_kernel(const int* __restrict__ prefix_len, int B, int
 void launch_mask_table(const int* prefix_len, int B, int T, int H, int* key_limit,
                        cudaStream_t s) {
   mask_table_kernel<<<(B * T + 255) / 256, 256, 0, s>>>(prefix_len, B, T, H, key_limit);
-}
-
-__global__ void row_gather_kernel(const uint8_t* src, uint8_t* dst, const int* perm,
-                                  int row_bytes) {
-  const int r = blockIdx.x;
-  const uint8_t* s = src + (size_t)perm[r] * row_bytes;
-  uint8_t* d = dst + (size_t)r * row_bytes;
-  for (int i = threadIdx.x * 16; i < row_bytes; i += blockDim.x * 16)
-    *reinterpret_cast<uint4*>(d + i) = *reinterpret_cast<const uint4*>(s + i);
-}
-
-void launch_row_gather(const void* src, void* dst, const int* perm, int rows, int row_bytes,
-                       cudaStream_t s) {
-  row_gather_kernel<<<rows, 128, 0, s>>>((const uint8_t*)src, (uint8_t*)dst, perm, row_bytes);
 }
 
 }  // namespace fva

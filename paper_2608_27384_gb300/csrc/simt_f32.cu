@@ -13,6 +13,8 @@ __global__ void __launch_bounds__(256) f32_gemm_kernel(const float* __restrict__
                                                        int N, int K) {
   __shared__ float sA[16][64 + 4];
   __shared__ float sB[16][64 + 4];
+  pdl_trigger();
+  pdl_wait();
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
   const int m0 = blockIdx.y * 64, n0 = blockIdx.x * 64;
   float acc[4][4] = {};
@@ -52,11 +54,13 @@ void launch_f32_gemm(const float* A, int lda, const float* B, float* C, int ldc,
                      int K, cudaStream_t s) {
   if (M <= 0) return;
   dim3 grid((N + 63) / 64, (M + 63) / 64);
-  f32_gemm_kernel<<<grid, 256, 0, s>>>(A, lda, B, C, ldc, M, N, K);
+  launch_pdl(f32_gemm_kernel, grid, dim3(256), 0, s, A, lda, B, C, ldc, M, N, K);
 }
 
 __global__ void f32_bias_act_kernel(const float* __restrict__ C, const float* __restrict__ bias,
                                     float* __restrict__ out, long long n, int N, bool silu) {
+  pdl_trigger();
+  pdl_wait();
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n;
        i += (long long)gridDim.x * blockDim.x) {
     const float v = C[i] + bias[i % N];
@@ -67,7 +71,8 @@ __global__ void f32_bias_act_kernel(const float* __restrict__ C, const float* __
 void launch_f32_bias_act(const float* C, const float* bias, float* out, int M, int N,
                          bool silu, cudaStream_t s) {
   if (M <= 0) return;
-  f32_bias_act_kernel<<<304, 256, 0, s>>>(C, bias, out, (long long)M * N, N, silu);
+  launch_pdl(f32_bias_act_kernel, dim3(304), dim3(256), 0, s, C, bias, out, (long long)M * N, N,
+             silu);
 }
 
 // C [M, nq*dh + 2*dh] = [q heads | k | v]; rotate q and k (rotate-half RoPE at
@@ -78,6 +83,8 @@ __global__ void f32_qkv_rope_kernel(const float* __restrict__ C, float* __restri
                                     const float2* __restrict__ rope, int T, int S_cap, int nq,
                                     int dh) {
   const int m = blockIdx.x, r = m / T, t = m % T;
+  pdl_trigger();
+  pdl_wait();
   const int pos = prefix_len[r] + t;
   const int half = dh / 2, N = (nq + 2) * dh;
   const float* row = C + (size_t)m * N;
@@ -101,12 +108,15 @@ void launch_f32_qkv_rope(const float* C, float* q, float* kc, float* vc,
                          const int* prefix_len, const float2* rope, int M, int T, int S_cap,
                          int nq, int dh, cudaStream_t s) {
   if (M <= 0) return;
-  f32_qkv_rope_kernel<<<M, 128, 0, s>>>(C, q, kc, vc, prefix_len, rope, T, S_cap, nq, dh);
+  launch_pdl(f32_qkv_rope_kernel, dim3(M), dim3(128), 0, s, C, q, kc, vc, prefix_len, rope, T,
+             S_cap, nq, dh);
 }
 
 // C [M, 2F] = [gate | up] -> out [M, F] = gelu_tanh(gate) * up.
 __global__ void f32_geglu_kernel(const float* __restrict__ C, float* __restrict__ out,
                                  long long n, int F) {
+  pdl_trigger();
+  pdl_wait();
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n;
        i += (long long)gridDim.x * blockDim.x) {
     const long long m = i / F, f = i % F;
@@ -116,7 +126,7 @@ __global__ void f32_geglu_kernel(const float* __restrict__ C, float* __restrict_
 
 void launch_f32_geglu(const float* C, float* out, int M, int F, cudaStream_t s) {
   if (M <= 0) return;
-  f32_geglu_kernel<<<304, 256, 0, s>>>(C, out, (long long)M * F, F);
+  launch_pdl(f32_geglu_kernel, dim3(304), dim3(256), 0, s, C, out, (long long)M * F, F);
 }
 
 // One CTA per (token row, head): softmax over the row's visible keys only.
@@ -127,6 +137,8 @@ __global__ void f32_attention_kernel(const float* __restrict__ q, const float* _
   extern __shared__ float sm[];  // [dh] query, then [limit] scores
   const int m = blockIdx.x, head = blockIdx.y;
   const int r = m / T, t = m % T;
+  pdl_trigger();
+  pdl_wait();
   const int P = prefix_len[r];
   const int limit = attn_key_limit(P, t, H);
   float* sq = sm;
@@ -178,8 +190,8 @@ void launch_f32_attention(const float* q, const float* kc, const float* vc,
   if (B * T <= 0) return;
   dim3 grid(B * T, nq);
   const size_t smem = sizeof(float) * (dh + max_keys);
-  f32_attention_kernel<<<grid, 128, smem, s>>>(q, kc, vc, prefix_len, out, T, H, nq, dh,
-                                               S_cap);
+  launch_pdl(f32_attention_kernel, grid, dim3(128), smem, s, q, kc, vc, prefix_len, out, T, H,
+             nq, dh, S_cap);
 }
 
 }  // namespace fva

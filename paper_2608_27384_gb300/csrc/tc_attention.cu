@@ -19,8 +19,8 @@
 //               keys, P = exp(S - max) written as bf16 into the swizzled A-operand
 //               layout in shared memory, row sum; then read O from TMEM.
 // A tile with one split writes O / l as bf16.  Otherwise each split writes its
-// (O, max, sum) to scratch and the last CTA of the tile (atomic ticket) merges
-// the splits in split order -- deterministic -- and writes bf16.
+// unnormalised (O, max, sum) to scratch and attn_merge_kernel combines the
+// splits of every row in split order (deterministic) and writes bf16.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -51,7 +51,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int limit_max = attn_key_limit(P, t_last, a.H);
   const int nkb_tile = (limit_max + kKB - 1) / kKB;
   const int nsplit = (nkb_tile + kBlocksPerSplit - 1) / kBlocksPerSplit;
-  if (split >= nsplit) return;  // uniform over the CTA, before any barrier / TMEM use
+  if (split >= nsplit) {  // uniform over the CTA, before any barrier / TMEM use
+    pdl_trigger();
+    return;
+  }
   const int kb0 = split * kBlocksPerSplit;
   const int nblk = min(kBlocksPerSplit, nkb_tile - kb0);
 
@@ -68,7 +71,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* p_full = bars + 6;
   uint64_t* o_full = bars + 7;
   uint32_t* tmem_slot = (uint32_t*)(bars + 8);
-  int* last_flag = (int*)(bars + 9);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -85,11 +87,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tmK);
     tma_prefetch_desc(&tmV);
   }
+  // Only one CTA of any tcgen05 kernel of this library fits on an SM (each uses
+  // more than half of the shared memory), so this allocation never waits.
   if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();  // q and the action K/V come from the QKV projection
   const uint32_t tS = tmem, tO = tmem + 256;
 
   const int qrow0 = (r * a.T + t0) * a.nq;
@@ -204,8 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_arrive(p_full);
     if (good) good = __all_sync(0xffffffffu, mbar_wait(o_full, 0, a.err, KERR_WAIT_MMA));
     tc_fence_after();
-    const int n_tiles_req = a.tiles_per_req;
-    const int gtile = r * n_tiles_req + tile;
+    const int gtile = r * a.tiles_per_req + tile;
     const int grow = qrow0 + row;  // global q row = (r*T + t) * nq + head
     if (good) {
       if (nsplit == 1) {
@@ -225,59 +230,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < kDH; c += 32) {
           float v[32];
           tmem_ld32(tO + lane_off + c, v);
+          if (!valid) continue;
 #pragma unroll
           for (int i = 0; i < 32; i += 4)
-            __stcg(reinterpret_cast<float4*>(po + c + i), make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]));
+            __stcg(reinterpret_cast<float4*>(po + c + i),
+                   make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]));
         }
-        __stcg(a.part_ml + ((size_t)gtile * a.max_splits + split) * kRows + row,
-               make_float2(mx, l));
-      }
-    }
-    if (nsplit > 1) {
-      // last-arriving split of this tile merges all splits in split order
-      __threadfence();
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      if (warp == 2 && lane == 0) {
-        const int ticket = atomicAdd(a.counters + gtile, 1);
-        *last_flag = (ticket == nsplit - 1) ? 1 : 0;
-        if (ticket == nsplit - 1) a.counters[gtile] = 0;  // ready for the next launch
-      }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      if (*last_flag) {
-        __threadfence();
-        if (valid) {
-          float m_all = -INFINITY;
-          for (int s = 0; s < nsplit; ++s) {
-            const float2 ml = __ldcg(a.part_ml + ((size_t)gtile * a.max_splits + s) * kRows + row);
-            if (ml.y > 0.f) m_all = fmaxf(m_all, ml.x);
-          }
-          float wsum = 0.f, wts[32];
-          const int ns = min(nsplit, 32);
-          for (int s = 0; s < ns; ++s) {
-            const float2 ml = __ldcg(a.part_ml + ((size_t)gtile * a.max_splits + s) * kRows + row);
-            const float w = ml.y > 0.f ? exp2f((ml.x - m_all) * a.scale_log2) : 0.f;
-            wts[s] = w;
-            wsum += w * ml.y;
-          }
-          const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
-          for (int c = 0; c < kDH; c += 8) {
-            float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-            for (int s = 0; s < ns; ++s) {
-              const float* po =
-                  a.part_o + (((size_t)gtile * a.max_splits + s) * kRows + row) * kDH + c;
-              const float4 x0 = __ldcg(reinterpret_cast<const float4*>(po));
-              const float4 x1 = __ldcg(reinterpret_cast<const float4*>(po + 4));
-              const float w = wts[s];
-              acc[0] = fmaf(w, x0.x, acc[0]); acc[1] = fmaf(w, x0.y, acc[1]);
-              acc[2] = fmaf(w, x0.z, acc[2]); acc[3] = fmaf(w, x0.w, acc[3]);
-              acc[4] = fmaf(w, x1.x, acc[4]); acc[5] = fmaf(w, x1.y, acc[5]);
-              acc[6] = fmaf(w, x1.z, acc[6]); acc[7] = fmaf(w, x1.w, acc[7]);
-            }
-#pragma unroll
-            for (int i = 0; i < 8; ++i) acc[i] *= inv;
-            *reinterpret_cast<uint4*>((bf16*)a.out + (size_t)grow * kDH + c) = pack_bf16x8(acc);
-          }
-        }
+        if (valid)
+          __stcg(a.part_ml + ((size_t)gtile * a.max_splits + split) * kRows + row,
+                 make_float2(mx, l));
       }
     }
   }
@@ -289,6 +250,48 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// Combine the key splits of every query row of tiles that have more than one:
+// o = sum_s 2^((m_s - m) c) O_s / sum_s 2^((m_s - m) c) l_s, m = max over splits
+// with keys, c = log2(e)/sqrt(dh); splits in order.  One warp per row, 8 dh
+// values per lane.
+__global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int gtile = blockIdx.x, r = blockIdx.y;
+  const int row = blockIdx.z * 8 + warp;
+  const int tok_per_tile = kRows / a.nq;
+  const int t0 = gtile * tok_per_tile;
+  pdl_trigger();
+  const int t_last = min(a.T, t0 + tok_per_tile) - 1;
+  const int t = t0 + row / a.nq;
+  if (t >= a.T) return;
+  pdl_wait();
+  const int P = __ldg(a.prefix_len + r);
+  const int nkb_tile = (attn_key_limit(P, t_last, a.H) + kKB - 1) / kKB;
+  const int nsplit = (nkb_tile + kBlocksPerSplit - 1) / kBlocksPerSplit;
+  if (nsplit <= 1) return;  // written directly by the attention kernel
+  const size_t tbase = (size_t)(r * a.tiles_per_req + gtile) * a.max_splits;
+  float2 ml = make_float2(-INFINITY, 0.f);
+  if (lane < nsplit) ml = __ldcg(a.part_ml + (tbase + lane) * kRows + row);
+  float m_all = warp_max(ml.y > 0.f ? ml.x : -INFINITY);
+  const float w = ml.y > 0.f ? exp2f((ml.x - m_all) * a.scale_log2) : 0.f;
+  const float inv = 1.f / warp_sum(w * ml.y);
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  for (int s = 0; s < nsplit; ++s) {
+    const float ws = __shfl_sync(0xffffffffu, w, s);
+    const float* po = a.part_o + ((tbase + s) * kRows + row) * kDH + lane * 8;
+    const float4 x0 = __ldcg(reinterpret_cast<const float4*>(po));
+    const float4 x1 = __ldcg(reinterpret_cast<const float4*>(po + 4));
+    acc[0] = fmaf(ws, x0.x, acc[0]); acc[1] = fmaf(ws, x0.y, acc[1]);
+    acc[2] = fmaf(ws, x0.z, acc[2]); acc[3] = fmaf(ws, x0.w, acc[3]);
+    acc[4] = fmaf(ws, x1.x, acc[4]); acc[5] = fmaf(ws, x1.y, acc[5]);
+    acc[6] = fmaf(ws, x1.z, acc[6]); acc[7] = fmaf(ws, x1.w, acc[7]);
+  }
+#pragma unroll
+  for (int i = 0; i < 8; ++i) acc[i] *= inv;
+  const size_t grow = (size_t)(r * a.T + t0) * a.nq + row;
+  *reinterpret_cast<uint4*>((bf16*)a.out + grow * kDH + lane * 8) = pack_bf16x8(acc);
+}
+
 }  // namespace
 
 cudaError_t tc_attention_init() {
@@ -298,10 +301,11 @@ cudaError_t tc_attention_init() {
 cudaError_t launch_tc_attention(const CUtensorMap* q, const CUtensorMap* k,
                                 const CUtensorMap* v, const AttnArgs& a, int B,
                                 cudaStream_t s) {
-  if (a.max_splits > 32) return cudaErrorInvalidValue;  // merge keeps <= 32 weights in registers
-  dim3 grid(a.tiles_per_req, a.max_splits, B);
-  tc_attn_kernel<<<grid, kThreads, kSmem, s>>>(*q, *k, *v, a);
-  return cudaGetLastError();
+  if (a.max_splits > 32) return cudaErrorInvalidValue;  // the merge holds one split per lane
+  cudaError_t e = launch_pdl(tc_attn_kernel, dim3(a.tiles_per_req, a.max_splits, B),
+                             dim3(kThreads), kSmem, s, *q, *k, *v, a);
+  if (e != cudaSuccess || a.max_splits == 1) return e;
+  return launch_pdl(attn_merge_kernel, dim3(a.tiles_per_req, B, kRows / 8), dim3(256), 0, s, a);
 }
 
 }  // namespace fva

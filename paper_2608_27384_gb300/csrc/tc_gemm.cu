@@ -154,11 +154,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
   }
+  // Only one CTA of any tcgen05 kernel of this library fits on an SM (each uses
+  // more than half of the shared memory), so this allocation never waits.
   if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();  // A (and the epilogue's destinations) belong to earlier kernels
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer
@@ -226,9 +230,8 @@ cudaError_t launch(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep
   const int kb_total = K / kBK;
   const int kbps = (kb_total + splits - 1) / splits;
   dim3 grid((M + kBM - 1) / kBM, N / BN, splits);
-  tc_gemm_kernel<BN, MODE><<<grid, kThreads, GemmCfg<BN>::kSmemBytes, s>>>(*a, *b, ep, M, N,
-                                                                            kb_total, kbps);
-  return cudaGetLastError();
+  return launch_pdl(tc_gemm_kernel<BN, MODE>, grid, dim3(kThreads), GemmCfg<BN>::kSmemBytes, s,
+                    *a, *b, ep, M, N, kb_total, kbps);
 }
 
 }  // namespace
