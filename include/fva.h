@@ -208,6 +208,27 @@ fva_status fva_get_step_index(const fva_handle* h, uint64_t* step);
  */
 fva_status fva_mask_table(fva_handle* h, int32_t batch, int32_t* key_limit, fva_stream stream);
 
+/*
+ * The chunk-wise causal multi-query attention of one expert layer (§3.1), as the
+ * step computes it, on caller-owned buffers (bf16 handles only):
+ *   q           device bf16 [batch*K*H*nq, head_dim]; row (r*K*H + t)*nq + head is
+ *               head `head` of action token t of request r (RoPE already applied).
+ *   k, v        device bf16 [batch, kv_rows, head_dim]: request r's keys/values in
+ *               the order [prefix_r ; action tokens 0..K*H-1].
+ *   prefix_len  device int32 [batch]: P_r, with P_r + K*H <= kv_rows.
+ *   out         device bf16 [batch*K*H*nq, head_dim] (same row order as q).
+ * Token t attends to the first P_r + (floor(t/H) + 1) H keys of its request;
+ * softmax scale 1/sqrt(head_dim).  Uses the handle's split-KV scratch, so calls
+ * on one handle must not overlap on the GPU.  Requires 1 <= batch <= max_batch and
+ * kv_rows <= max_prefix + K*H, and 16-byte aligned pointers.  Errors: INVALID_ARG,
+ * UNSUPPORTED (fp32 handle), CUDA.  A device P_r that breaks P_r + K*H <= kv_rows
+ * cannot be seen on the host: the kernel leaves those rows unwritten and the
+ * next fva_step on the handle returns FVA_ERR_INVALID_ARG.
+ */
+fva_status fva_chunk_attention(fva_handle* h, const void* q, const void* k, const void* v,
+                               const int32_t* prefix_len, int32_t batch, int32_t kv_rows,
+                               void* out, fva_stream stream);
+
 /* Kernels of one step, as reported by fva_step_profile. */
 typedef enum fva_kernel_kind {
   FVA_K_TIMESTEP_EMBED = 0,  /* sinusoidal embedding of every chunk's tau             */

@@ -64,7 +64,7 @@ KERNEL_KINDS = ["timestep_embed", "time_mlp", "film", "embed_norm", "qkv", "atte
 EXPORTS = ["fva_create", "fva_destroy", "fva_num_weights", "fva_weight_shape",
            "fva_load_weights", "fva_set_prefix_kv", "fva_step", "fva_step_ex",
            "fva_trace_floats", "fva_set_step_index", "fva_get_step_index", "fva_mask_table",
-           "fva_step_profile", "fva_last_error"]
+           "fva_step_profile", "fva_chunk_attention", "fva_last_error"]
 
 _lib_handle: Optional[ctypes.CDLL] = None
 
@@ -95,6 +95,7 @@ def lib() -> ctypes.CDLL:
         "fva_mask_table": (i32, [vp, i32, vp, vp]),
         "fva_step_profile": (i32, [vp, vp, P(ctypes.c_float), vp, i32, P(fva_kernel_time), i32,
                                    P(i32), vp]),
+        "fva_chunk_attention": (i32, [vp, vp, vp, vp, vp, i32, i32, vp, vp]),
         "fva_last_error": (ctypes.c_char_p, []),
     }
     for name, (res, args) in sig.items():
@@ -223,3 +224,9 @@ def fva_step_profile(handle: int, buffer, noise_levels, out_chunk, batch: int, s
                                   ctypes.byref(n), _stream(stream)))
     return [(KERNEL_KINDS[recs[i].kind], recs[i].layer, recs[i].microseconds)
             for i in range(n.value)]
+
+
+def fva_chunk_attention(handle: int, q, k, v, prefix_len, batch: int, kv_rows: int, out,
+                        stream=None) -> None:
+    _check(lib().fva_chunk_attention(handle, _ptr(q), _ptr(k), _ptr(v), _ptr(prefix_len), batch,
+                                     kv_rows, _ptr(out), _stream(stream)))

@@ -22,6 +22,7 @@ enum : int {
   KERR_WAIT_TMA = 1,   // a consumer waited too long for a TMA load
   KERR_WAIT_MMA = 2,   // a producer/epilogue waited too long for the tensor core
   KERR_WAIT_SYNC = 3,  // softmax/epilogue hand-off timed out
+  KERR_BAD_SHAPE = 4,  // a device-side size (e.g. a prefix length) broke a kernel bound
 };
 
 // Wall-clock bound of every spin-wait (ns).  Far above any legitimate wait.

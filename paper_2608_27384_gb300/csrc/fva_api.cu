@@ -902,9 +902,12 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
 fva_status check_async_error(fva_handle* h) {
   if (h->err_pending && cudaEventQuery(h->err_ev) == cudaSuccess) {
     h->err_pending = false;
-    if (*h->err_host != 0)
+    const int code = *h->err_host;
+    if (code == 4 /* KERR_BAD_SHAPE */)
+      return fail(FVA_ERR_INVALID_ARG, "an earlier kernel saw a device size beyond its bound");
+    if (code != 0)
       return fail(FVA_ERR_TIMEOUT, "a kernel of an earlier step gave up a bounded wait (code %d)",
-                  *h->err_host);
+                  code);
   }
   cudaError_t e = cudaPeekAtLastError();
   if (e != cudaSuccess && e != cudaErrorNotReady) {
@@ -1100,5 +1103,47 @@ extern "C" fva_status fva_mask_table(fva_handle* h, int32_t batch, int32_t* key_
   DeviceGuard guard(h->device);
   launch_mask_table(h->prefix_len_dev, batch, h->T, h->H, key_limit, (cudaStream_t)stream);
   CUDA_TRY(cudaGetLastError());
+  return FVA_OK;
+}
+
+// =============================================================================
+// isolated chunk-causal attention on caller buffers
+// =============================================================================
+extern "C" fva_status fva_chunk_attention(fva_handle* h, const void* q, const void* k,
+                                          const void* v, const int32_t* prefix_len,
+                                          int32_t batch, int32_t kv_rows, void* out,
+                                          fva_stream stream) {
+  if (!h || !q || !k || !v || !prefix_len || !out) return fail(FVA_ERR_INVALID_ARG, "NULL argument");
+  if (!h->bf16) return fail(FVA_ERR_UNSUPPORTED, "fva_chunk_attention needs a bf16 handle");
+  if (batch < 1 || batch > h->Bmax)
+    return fail(FVA_ERR_INVALID_ARG, "batch %d outside [1, %d]", batch, h->Bmax);
+  if (kv_rows < h->T || kv_rows > h->S_cap)
+    return fail(FVA_ERR_INVALID_ARG, "kv_rows %d outside [K*H, max_prefix + K*H] = [%d, %d]",
+                kv_rows, h->T, h->S_cap);
+  for (const void* p : {q, k, v, (const void*)out})
+    if (reinterpret_cast<uintptr_t>(p) % 16)
+      return fail(FVA_ERR_INVALID_ARG, "q, k, v and out must be 16-byte aligned");
+  DeviceGuard guard(h->device);
+  fva_status st;
+  CUtensorMap mq, mk, mv;
+  if ((st = make_map(&mq, q, (uint64_t)batch * h->T * h->nq, h->dh, 128)) ||
+      (st = make_map(&mk, k, (uint64_t)batch * kv_rows, h->dh, 64)) ||
+      (st = make_map(&mv, v, (uint64_t)batch * kv_rows, h->dh, 64)))
+    return st;
+  AttnArgs aa{};
+  aa.prefix_len = prefix_len;
+  aa.out = out;
+  aa.part_o = h->att_part_o;
+  aa.part_ml = h->att_part_ml;
+  aa.T = h->T;
+  aa.H = h->H;
+  aa.nq = h->nq;
+  aa.S_cap = kv_rows;
+  aa.tiles_per_req = h->tiles_per_req;
+  aa.max_splits = (kv_rows + kAttnKeysPerSplit - 1) / kAttnKeysPerSplit;
+  aa.kv_row0 = 0;
+  aa.scale_log2 = 1.4426950408889634f / std::sqrt((float)h->dh);
+  aa.err = h->err_dev;
+  CUDA_TRY(launch_tc_attention(&mq, &mk, &mv, aa, batch, (cudaStream_t)stream));
   return FVA_OK;
 }

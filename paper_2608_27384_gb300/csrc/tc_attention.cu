@@ -51,7 +51,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int limit_max = attn_key_limit(P, t_last, a.H);
   const int nkb_tile = (limit_max + kKB - 1) / kKB;
   const int nsplit = (nkb_tile + kBlocksPerSplit - 1) / kBlocksPerSplit;
-  if (split >= nsplit) {  // uniform over the CTA, before any barrier / TMEM use
+  if (split >= nsplit || nsplit > a.max_splits) {  // uniform over the CTA
+    if (nsplit > a.max_splits && split == 0 && threadIdx.x == 0) report_error(a.err, KERR_BAD_SHAPE);
     pdl_trigger();
     return;
   }
@@ -268,7 +269,7 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
   const int P = __ldg(a.prefix_len + r);
   const int nkb_tile = (attn_key_limit(P, t_last, a.H) + kKB - 1) / kKB;
   const int nsplit = (nkb_tile + kBlocksPerSplit - 1) / kBlocksPerSplit;
-  if (nsplit <= 1) return;  // written directly by the attention kernel
+  if (nsplit <= 1 || nsplit > a.max_splits) return;  // written by the attention kernel / bad size
   const size_t tbase = (size_t)(r * a.tiles_per_req + gtile) * a.max_splits;
   float2 ml = make_float2(-INFINITY, 0.f);
   if (lane < nsplit) ml = __ldcg(a.part_ml + (tbase + lane) * kRows + row);
