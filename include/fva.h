@@ -229,6 +229,34 @@ fva_status fva_chunk_attention(fva_handle* h, const void* q, const void* k, cons
                                const int32_t* prefix_len, int32_t batch, int32_t kv_rows,
                                void* out, fva_stream stream);
 
+/*
+ * fva_chunk_attention without any device allocation and without a handle.  The
+ * paper has no counterpart: this exists for callers that cannot allocate device
+ * memory -- a controller running the decoder in a fixed-period loop, where
+ * cudaMalloc / cudaFree may synchronise the device for an unbounded time, or a
+ * host that gives all device memory to its own pool at start-up.
+ *
+ * Same inputs, output and numerics as fva_chunk_attention, with the shapes passed
+ * explicitly (head_dim must be 256, n_q_heads one of 1, 2, 4, 8, 16).  The split-KV
+ * scratch is a fixed array inside the library: 256 slots of 128 x 256 fp32 plus
+ * row statistics (32 MiB + 256 KiB), kept by every GPU that loads the library
+ * until the process exits.  A call needs
+ *   batch * ceil(K*H*n_q_heads / 128) * ceil(kv_rows / 256)
+ * slots (and ceil(kv_rows / 256) <= 32); larger calls return FVA_ERR_INVALID_ARG.
+ * The first call on a device looks up the array's device address (and sets the
+ * kernel attributes) with that device current; make that first call before any
+ * stream capture.  Every call uses the same array, which keeps the last call's
+ * contents (nothing in it needs to start at zero): calls that overlap on the GPU,
+ * from any thread or stream, race.  Device-side problems (a prefix length beyond
+ * kv_rows - K*H) leave the affected rows unwritten and are not reported.
+ * Calls no cudaMalloc, cudaFree or other allocating routine.
+ */
+fva_status fva_chunk_attention_noalloc(const void* q, const void* k, const void* v,
+                                       const int32_t* prefix_len, int32_t batch,
+                                       int32_t n_chunks, int32_t chunk_tokens,
+                                       int32_t n_q_heads, int32_t head_dim, int32_t kv_rows,
+                                       void* out, fva_stream stream);
+
 /* Kernels of one step, as reported by fva_step_profile. */
 typedef enum fva_kernel_kind {
   FVA_K_TIMESTEP_EMBED = 0,  /* sinusoidal embedding of every chunk's tau             */

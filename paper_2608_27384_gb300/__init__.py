@@ -64,7 +64,8 @@ KERNEL_KINDS = ["timestep_embed", "time_mlp", "film", "embed_norm", "qkv", "atte
 EXPORTS = ["fva_create", "fva_destroy", "fva_num_weights", "fva_weight_shape",
            "fva_load_weights", "fva_set_prefix_kv", "fva_step", "fva_step_ex",
            "fva_trace_floats", "fva_set_step_index", "fva_get_step_index", "fva_mask_table",
-           "fva_step_profile", "fva_chunk_attention", "fva_last_error"]
+           "fva_step_profile", "fva_chunk_attention", "fva_chunk_attention_noalloc",
+           "fva_last_error"]
 
 _lib_handle: Optional[ctypes.CDLL] = None
 
@@ -96,6 +97,8 @@ def lib() -> ctypes.CDLL:
         "fva_step_profile": (i32, [vp, vp, P(ctypes.c_float), vp, i32, P(fva_kernel_time), i32,
                                    P(i32), vp]),
         "fva_chunk_attention": (i32, [vp, vp, vp, vp, vp, i32, i32, vp, vp]),
+        "fva_chunk_attention_noalloc": (i32, [vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, vp,
+                                              vp]),
         "fva_last_error": (ctypes.c_char_p, []),
     }
     for name, (res, args) in sig.items():
@@ -230,3 +233,12 @@ def fva_chunk_attention(handle: int, q, k, v, prefix_len, batch: int, kv_rows: i
                         stream=None) -> None:
     _check(lib().fva_chunk_attention(handle, _ptr(q), _ptr(k), _ptr(v), _ptr(prefix_len), batch,
                                      kv_rows, _ptr(out), _stream(stream)))
+
+
+def fva_chunk_attention_noalloc(q, k, v, prefix_len, batch: int, n_chunks: int,
+                                chunk_tokens: int, n_q_heads: int, head_dim: int, kv_rows: int,
+                                out, stream=None) -> None:
+    """fva_chunk_attention with the library's fixed scratch: allocates nothing."""
+    _check(lib().fva_chunk_attention_noalloc(_ptr(q), _ptr(k), _ptr(v), _ptr(prefix_len), batch,
+                                             n_chunks, chunk_tokens, n_q_heads, head_dim,
+                                             kv_rows, _ptr(out), _stream(stream)))

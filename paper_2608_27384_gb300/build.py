@@ -18,7 +18,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libfva.so")
 
-SOURCES = ["fva_api.cu", "rowwise.cu", "tc_gemm.cu", "tc_attention.cu", "simt_f32.cu"]
+SOURCES = ["fva_api.cu", "rowwise.cu", "tc_gemm.cu", "tc_attention.cu", "simt_f32.cu",
+           "attention_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -431,6 +431,8 @@ extern "C" void fva_destroy(fva_handle* h) {
 
 extern "C" const char* fva_last_error(void) { return g_last_error.c_str(); }
 
+void fva::set_last_error(const char* msg) { g_last_error = msg; }
+
 // =============================================================================
 // weights
 // =============================================================================

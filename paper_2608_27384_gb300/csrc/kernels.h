@@ -35,6 +35,9 @@ __host__ __device__ __forceinline__ int modf_off(int L, int which, int W) {
   return L * 6 * W + which * W;
 }
 
+// Sets the text fva_last_error() returns on the calling thread (fva_api.cu).
+void set_last_error(const char* msg);
+
 // ---------------------------------------------------------------- rowwise.cu
 // act_bf16 selects the activation type (bf16 when true, else fp32).
 void launch_temb(const float* tau, int rows, int W, float tmin, float tmax, void* out,
