@@ -81,7 +81,11 @@ def kernel_costs(wl, B):
     c["time_mlp"] = (2.0 * BK * W * W, 2.0 * W * W)
     c["resid_norm"] = (0.0, 4.0 * M * W * 3 + 2.0 * M * W)
     c["embed_norm"] = (2.0 * M * A * W, 4.0 * M * (A + W) + 2.0 * M * W)
-    c["final"] = (2.0 * M * W * A, 4.0 * M * W * 2 + 4.0 * M * A * 3)
+    c["final_norm"] = (0.0, 4.0 * M * W * 3 + 4.0 * M * W)
+    c["velocity"] = (2.0 * M * W * A, 4.0 * M * W + 4.0 * W * A + 4.0 * M * A * 3)
+    tiles = -(-T * nq // 128)
+    c["attn_merge"] = (0.0, 4.0 * B * tiles * 128 * dh * max(1, -(-(max(P) + T) // 256)) +
+                       2.0 * M * Dq)
     c["timestep_embed"] = (0.0, 2.0 * BK * W)
     return c
 
@@ -92,7 +96,7 @@ def step_costs(wl, B):
     L = wl.n_layers
     c = kernel_costs(wl, B)
     flops = L * sum(c[k][0] for k in ("qkv", "out_proj", "gate_up", "down", "attention"))
-    flops += c["film"][0] + 2 * c["time_mlp"][0] + c["embed_norm"][0] + c["final"][0]
+    flops += c["film"][0] + 2 * c["time_mlp"][0] + c["embed_norm"][0] + c["velocity"][0]
     W, F, Dq, dh, A = wl.width, wl.mlp_dim, wl.n_q_heads * wl.head_dim, wl.head_dim, wl.action_dim
     wbytes = 2.0 * L * ((Dq + 2 * dh) * W + W * Dq + 2 * F * W + W * F)
     wbytes += 2.0 * (L * 6 * W + 2 * W) * W + 2.0 * 2 * W * W + 4.0 * 2 * A * W

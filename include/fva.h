@@ -269,8 +269,10 @@ typedef enum fva_kernel_kind {
   FVA_K_RESID_NORM = 7,      /* split-K reduction + gated residual + FiLM RMSNorm    */
   FVA_K_GATE_UP = 8,         /* packed gate/up projection + tanh-GELU gating         */
   FVA_K_DOWN = 9,            /* MLP down projection (split-K partials)               */
-  FVA_K_FINAL = 10,          /* final norm + out-projection + Euler + emit + roll    */
-  FVA_K_COUNT = 11
+  FVA_K_FINAL = 10,          /* last gated residual + final FiLM RMSNorm (fp32 out)  */
+  FVA_K_ATTN_MERGE = 11,     /* combination of the attention's key splits            */
+  FVA_K_VELOCITY = 12,       /* out-projection + Euler + emit + roll + tail          */
+  FVA_K_COUNT = 13
 } fva_kernel_kind;
 
 typedef struct fva_kernel_time {

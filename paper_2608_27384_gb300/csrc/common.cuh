@@ -114,6 +114,17 @@ __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 
+// Plain bulk copy global -> shared (both 16-byte aligned, bytes a multiple of
+// 16), completing on `bar` with complete_tx.
+__device__ __forceinline__ void bulk_load(void* smem_dst, const void* gsrc, uint32_t bytes,
+                                          uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(smem_dst)),
+      "l"(gsrc), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
 __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* map, int32_t x,
                                             int32_t y, uint64_t* bar) {
   asm volatile(
@@ -121,6 +132,38 @@ __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* m
       " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_u32(smem_dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar))
       : "memory");
+}
+
+// Ask the memory system to bring [addr, addr + bytes) into L2 (fire and forget).
+// addr and bytes must be multiples of 16.
+__device__ __forceinline__ void prefetch_l2_bulk(const void* addr, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(addr), "r"(bytes) : "memory");
+}
+
+// Up to three byte ranges to prefetch into L2, split into 64 KiB pieces that the
+// CTAs of a grid issue round-robin (thread 0 of each CTA).
+struct L2Prefetch {
+  const void* ptr[3];
+  unsigned long long bytes[3];
+};
+
+__device__ __forceinline__ void issue_l2_prefetch(const L2Prefetch& pf) {
+  if (threadIdx.x != 0) return;
+  constexpr unsigned long long kPiece = 65536;
+  unsigned long long base = 0;
+  for (int r = 0; r < 3; ++r) {
+    const unsigned long long n = pf.bytes[r];
+    if (!pf.ptr[r] || n == 0) continue;
+    const unsigned long long pieces = (n + kPiece - 1) / kPiece;
+    // piece i of this range has global index base + i; CTA b takes indices = b mod grid
+    unsigned long long first = (blockIdx.x + gridDim.x - base % gridDim.x) % gridDim.x;
+    for (unsigned long long i = first; i < pieces; i += gridDim.x) {
+      const unsigned long long off = i * kPiece;
+      const unsigned long long len = (n - off < kPiece) ? (n - off) : kPiece;
+      prefetch_l2_bulk((const uint8_t*)pf.ptr[r] + off, (uint32_t)(len & ~15ull));
+    }
+    base += pieces;
+  }
 }
 
 // ----------------------------------------------------------------------------
@@ -191,6 +234,25 @@ __device__ __forceinline__ void umma_commit(uint64_t* bar) {
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
           smem_u32(bar))
       : "memory");
+}
+
+// 32 consecutive fp32 columns of this thread's TMEM lane, without waiting:
+// call tmem_ld_wait() before using any of the values (several loads may be in
+// flight at once).
+__device__ __forceinline__ void tmem_ld32_nowait(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
 // 32 consecutive fp32 columns of this thread's TMEM lane.

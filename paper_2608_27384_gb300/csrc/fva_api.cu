@@ -14,6 +14,7 @@
 #include <string>
 #include <vector>
 
+#include "common.cuh"
 #include "fva.h"
 #include "kernels.h"
 
@@ -131,7 +132,7 @@ struct fva_handle {
   void* warena = nullptr;
   size_t warena_bytes = 0;
   float *w_in_t = nullptr, *b_in = nullptr, *b_t1 = nullptr, *b_t2 = nullptr, *b_mod = nullptr;
-  float *w_out = nullptr, *b_out = nullptr;
+  float *w_out_t = nullptr, *b_out = nullptr;  // w_out_t: [W, A]
   void *w_t1 = nullptr, *w_t2 = nullptr, *w_mod = nullptr;
   std::vector<LayerW> layers;
   CUtensorMap m_wt1, m_wt2, m_wmod;
@@ -141,10 +142,12 @@ struct fva_handle {
   int* prefix_len_dev = nullptr;
   std::vector<int> layer_len;  // [Bmax * L], -1 = never set
   float2* rope = nullptr;
+  float2* temb_freq = nullptr;  // [W/2] two-float split of 2 / p_j
   // activations / scratch
   void *temb = nullptr, *t1 = nullptr, *cond = nullptr, *y = nullptr, *q = nullptr;
   void *attn = nullptr, *mlp = nullptr;
   float *mod = nullptr, *h = nullptr, *part = nullptr, *c32 = nullptr, *vel = nullptr;
+  float* yF = nullptr;  // [Mmax, W] fp32 output of the final FiLM RMSNorm
   float* fresh = nullptr;
   float* att_part_o = nullptr;
   float2* att_part_ml = nullptr;
@@ -328,6 +331,8 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
     if ((st = get_encoder()) != FVA_OK) return st;
     CUDA_TRY(tc_gemm_init());
     CUDA_TRY(tc_attention_init());
+    if (h->W > 4096) return fail(FVA_ERR_UNSUPPORTED, "bf16 kernels need width <= 4096");
+    CUDA_TRY(gemv_init(h->W));
   }
   const size_t a = h->act;
   const size_t kv_elems = (size_t)h->L * h->Bmax * h->S_cap * h->dh;
@@ -344,6 +349,7 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
       (st = dalloc(h, &h->attn, (size_t)h->Mmax * h->Dq, a)) ||
       (st = dalloc(h, &h->mlp, (size_t)h->Mmax * h->F, a)) ||
       (st = dalloc(h, &h->vel, (size_t)h->Mmax * h->A)) ||
+      (st = dalloc(h, &h->yF, (size_t)h->Mmax * h->W)) ||
       (st = dalloc(h, &h->fresh, (size_t)h->Bmax * h->H * h->A)) ||
       (st = dalloc(h, &h->err_dev, 1)))
     return st;
@@ -379,8 +385,32 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
   for (auto& e : h->ring_ev) CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
   CUDA_TRY(cudaEventCreateWithFlags(&h->err_ev, cudaEventDisableTiming));
   CUDA_TRY(cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking));
+  {
+    StepDims d{};
+    d.K = h->K;
+    d.A = h->A;
+    d.W = h->W;
+    if (sizeof(float) * ((size_t)2 * d.K * d.A + (size_t)(d.K + d.A) * 4) > 200 * 1024)
+      return fail(FVA_ERR_UNSUPPORTED, "n_chunks * action_dim too large for the final kernel");
+    CUDA_TRY(final_init(d));
+  }
   launch_rope_table(h->rope, h->S_cap, h->dh, c.rope_theta, 0);
   CUDA_TRY(cudaGetLastError());
+  {
+    // 2 / p_j in half turns per unit tau, p_j = t_min (t_max / t_min)^(j / (W/2 - 1))
+    const int half = h->W / 2;
+    std::vector<float2> fq(half);
+    for (int j = 0; j < half; ++j) {
+      const double period = (double)c.t_min_period *
+                            std::pow((double)c.t_max_period / (double)c.t_min_period,
+                                     half > 1 ? (double)j / (double)(half - 1) : 0.0);
+      const double v = 2.0 / period;
+      const float hi = (float)v;
+      fq[j] = make_float2(hi, (float)(v - (double)hi));
+    }
+    if ((st = dalloc(h, &h->temb_freq, half))) return st;
+    CUDA_TRY(cudaMemcpy(h->temb_freq, fq.data(), sizeof(float2) * half, cudaMemcpyHostToDevice));
+  }
   if (h->bf16) {
     const uint64_t M = h->Mmax, BK = h->BKmax;
     if ((st = make_map(&h->m_temb, h->temb, BK, h->W, 128)) ||
@@ -524,7 +554,10 @@ extern "C" fva_status fva_load_weights(fva_handle* h, const void* const* tensors
   const size_t o_bt1 = f32_off(t[3].data(), W);
   const size_t o_bt2 = f32_off(t[5].data(), W);
   const size_t o_bmod = f32_off(b_mod.data(), b_mod.size());
-  const size_t o_wout = f32_off(t[fin + 2].data(), (size_t)A * W);
+  std::vector<float> w_out_t((size_t)W * A);  // [W, A]
+  for (int a2 = 0; a2 < A; ++a2)
+    for (int w = 0; w < W; ++w) w_out_t[(size_t)w * A + a2] = t[fin + 2][(size_t)a2 * W + w];
+  const size_t o_wout = f32_off(w_out_t.data(), (size_t)A * W);
   const size_t o_bout = f32_off(t[fin + 3].data(), A);
 
   // matrices in the activation dtype, laid out for the kernels.
@@ -609,7 +642,7 @@ extern "C" fva_status fva_load_weights(fva_handle* h, const void* const* tensors
   h->b_t1 = fb + o_bt1;
   h->b_t2 = fb + o_bt2;
   h->b_mod = fb + o_bmod;
-  h->w_out = fb + o_wout;
+  h->w_out_t = fb + o_wout;
   h->b_out = fb + o_bout;
   h->w_t1 = base + o_wt1;
   h->w_t2 = base + o_wt2;
@@ -749,19 +782,14 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
 
   // ---- per-chunk FiLM condition and modulation (App. A.4)
   mark(FVA_K_TIMESTEP_EMBED, -1);
-  launch_temb(h->tau_dev(), BK, W, h->cfg.t_min_period, h->cfg.t_max_period, h->temb, bf, s);
+  launch_temb(h->tau_dev(), h->temb_freq, BK, W, h->temb, bf, s);
   GemmEpi ep{};
   ep.err = h->err_dev;
   if (bf) {
-    ep.out = h->t1;
-    ep.bias = h->b_t1;
-    ep.ldo = W;
     mark(FVA_K_TIME_MLP, -1);
-    CUDA_TRY(launch_tc_gemm(kBnTime, GEMM_BIAS_SILU_BF16, &h->m_temb, &h->m_wt1, ep, BK, W, W, 1, s));
-    ep.out = h->cond;
-    ep.bias = h->b_t2;
+    launch_gemv_silu(h->temb, h->w_t1, h->b_t1, h->t1, BK, W, W, s);
     mark(FVA_K_TIME_MLP, -1);
-    CUDA_TRY(launch_tc_gemm(kBnTime, GEMM_BIAS_SILU_BF16, &h->m_t1, &h->m_wt2, ep, BK, W, W, 1, s));
+    launch_gemv_silu(h->t1, h->w_t2, h->b_t2, h->cond, BK, W, W, s);
     ep.out = h->mod;
     ep.bias = h->b_mod;
     ep.ldo = h->N_mod;
@@ -779,8 +807,34 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
 
   // ---- action in-projection + layer 0 norm 1
   mark(FVA_K_EMBED_NORM, -1);
-  launch_embed_norm(d, buffer, h->w_in_t, h->b_in, h->mod, h->h, h->y, bf, s);
+  {
+    L2Prefetch pf0{};
+    const LayerW& lw = h->layers[0];
+    pf0.ptr[0] = lw.w_qkv;
+    pf0.bytes[0] = (unsigned long long)((const uint8_t*)lw.w_d - (const uint8_t*)lw.w_qkv) +
+                   (unsigned long long)W * F * a;
+    pf0.ptr[1] = h->kc;
+    pf0.bytes[1] = (size_t)B * h->S_cap * h->dh * a;
+    pf0.ptr[2] = h->vc;
+    pf0.bytes[2] = pf0.bytes[1];
+    launch_embed_norm(d, buffer, h->w_in_t, h->b_in, h->mod, h->h, h->y, bf, &pf0, s);
+  }
 
+  // L2 prefetch of layer l's weights and prefix/action K/V, issued by the norm
+  // kernel that precedes the layer (it runs while the previous GEMM drains).
+  const size_t kv_bytes_layer = (size_t)B * h->S_cap * h->dh * a;
+  auto layer_prefetch = [&](int l) {
+    L2Prefetch pf{};
+    const LayerW& lw = h->layers[l];
+    pf.ptr[0] = lw.w_qkv;
+    pf.bytes[0] = (unsigned long long)((const uint8_t*)lw.w_d - (const uint8_t*)lw.w_qkv) +
+                  (unsigned long long)W * F * a;
+    pf.ptr[1] = (const uint8_t*)h->kc + (size_t)l * kv_layer * a;
+    pf.bytes[1] = kv_bytes_layer;
+    pf.ptr[2] = (const uint8_t*)h->vc + (size_t)l * kv_layer * a;
+    pf.bytes[2] = kv_bytes_layer;
+    return pf;
+  };
   const int m_tiles = (M + 127) / 128;
   const int sp_o = bf ? choose_splits(m_tiles * (W / kBnResid), Dq / 64) : 1;
   const int sp_d = bf ? choose_splits(m_tiles * (W / kBnResid), F / 64) : 1;
@@ -838,6 +892,10 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       aa.err = h->err_dev;
       mark(FVA_K_ATTENTION, l);
       CUDA_TRY(launch_tc_attention(&h->m_q, &h->m_k, &h->m_v, aa, B, s));
+      if (aa.max_splits > 1) {
+        mark(FVA_K_ATTN_MERGE, l);
+        CUDA_TRY(launch_attn_merge(aa, B, s));
+      }
     } else {
       launch_f32_attention((float*)h->q, (float*)kc_l, (float*)vc_l, h->prefix_len_dev,
                            (float*)h->attn, B, h->T, h->H, h->nq, h->dh, h->S_cap, h->S_cap, s);
@@ -857,7 +915,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     }
     mark(FVA_K_RESID_NORM, l);
     launch_resid_norm(d, h->h, h->part, sp_o, pstride, h->mod, mod_off(l, 2, W), mod_off(l, 3, W),
-                      mod_off(l, 4, W), h->y, bf, s);
+                      mod_off(l, 4, W), h->y, bf, nullptr, s);
     if (trace) {
       CUDA_TRY(copy_h(o_hmid));
       launch_to_f32(h->y, bf, tr_at(o_y2), (long long)MW, s);
@@ -883,16 +941,18 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     if (trace) launch_to_f32(h->mlp, bf, tr_at(o_mlp), (long long)M * F, s);
     if (l + 1 < L) {
       mark(FVA_K_RESID_NORM, l);
+      const L2Prefetch pf = layer_prefetch(l + 1);
       launch_resid_norm(d, h->h, h->part, sp_d, pstride, h->mod, mod_off(l, 5, W),
-                        mod_off(l + 1, 0, W), mod_off(l + 1, 1, W), h->y, bf, s);
+                        mod_off(l + 1, 0, W), mod_off(l + 1, 1, W), h->y, bf, &pf, s);
       if (trace) CUDA_TRY(copy_h(o_hout));
     }
   }
   // ---- final norm, out-projection, Euler update, emit, roll, tail
   mark(FVA_K_FINAL, -1);
-  launch_final(d, h->h, h->part, sp_d, pstride, h->mod, h->w_out, h->b_out, h->dt_dev(), buffer,
-               out_chunk, h->vel, use_fresh ? h->fresh : nullptr, h->cfg.noise_seed,
-               h->step_dev(), s);
+  launch_final_norm(d, h->h, h->part, sp_d, pstride, h->mod, h->yF, s);
+  mark(FVA_K_VELOCITY, -1);
+  launch_velocity_euler(d, h->yF, h->w_out_t, h->b_out, h->dt_dev(), buffer, out_chunk, h->vel,
+                        use_fresh ? h->fresh : nullptr, h->cfg.noise_seed, h->step_dev(), s);
   if (tr.layer == L - 1) CUDA_TRY(copy_h(o_hout));
   mark(FVA_K_COUNT, -1);
   CUDA_TRY(cudaGetLastError());
@@ -1063,7 +1123,7 @@ extern "C" fva_status fva_step_profile(fva_handle* h, float* buffer, const float
   if (!records || !n_records) return fail(FVA_ERR_INVALID_ARG, "records / n_records is NULL");
   *n_records = 0;
   if (h) {
-    const int needed = 5 + 7 * h->L;
+    const int needed = 6 + 8 * h->L;
     if (max_records < needed)
       return fail(FVA_ERR_INVALID_ARG, "max_records %d < %d launches", max_records, needed);
   }
@@ -1147,5 +1207,6 @@ extern "C" fva_status fva_chunk_attention(fva_handle* h, const void* q, const vo
   aa.scale_log2 = 1.4426950408889634f / std::sqrt((float)h->dh);
   aa.err = h->err_dev;
   CUDA_TRY(launch_tc_attention(&mq, &mk, &mv, aa, batch, (cudaStream_t)stream));
+  CUDA_TRY(launch_attn_merge(aa, batch, (cudaStream_t)stream));
   return FVA_OK;
 }

@@ -40,24 +40,41 @@ void set_last_error(const char* msg);
 
 // ---------------------------------------------------------------- rowwise.cu
 // act_bf16 selects the activation type (bf16 when true, else fp32).
-void launch_temb(const float* tau, int rows, int W, float tmin, float tmax, void* out,
+// freq[j] = (hi, lo) two-float split of 2 / p_j, j < W/2 (see temb_kernel).
+void launch_temb(const float* tau, const float2* freq, int rows, int W, void* out,
                  bool act_bf16, cudaStream_t s);
 
+struct L2Prefetch;
+
+// pf (nullable): byte ranges the kernel's CTAs prefetch into L2 before waiting
+// on their predecessor (the next layer's weights and prefix K/V).
 void launch_embed_norm(const StepDims& d, const float* buffer, const float* w_in_t,
                        const float* b_in, const float* mod, float* h, void* y, bool act_bf16,
-                       cudaStream_t s);
+                       const L2Prefetch* pf, cudaStream_t s);
 
 // h += gate * sum_z part[z];  y = rmsnorm(h) * (1 + scale) + shift.
 void launch_resid_norm(const StepDims& d, float* h, const float* part, int n_parts,
                        long long part_stride, const float* mod, int gate_off, int scale_off,
-                       int shift_off, void* y, bool act_bf16, cudaStream_t s);
+                       int shift_off, void* y, bool act_bf16, const L2Prefetch* pf,
+                       cudaStream_t s);
 
-// Final residual, final norm, out-projection, Euler update, emit, roll, tail.
-void launch_final(const StepDims& d, float* h, const float* part, int n_parts,
-                  long long part_stride, const float* mod, const float* w_out,
-                  const float* b_out, const float* dt, float* buffer, float* out_chunk,
-                  float* vel_out, const float* fresh, unsigned long long seed,
-                  const unsigned long long* step_idx, cudaStream_t s);
+// Final residual + final FiLM RMSNorm (fp32 y_F into yF [B*K*H, W]), then
+// out-projection, Euler update, emit, roll and tail (two launches).  w_out_t is
+// W_out transposed, [W, A] fp32.  final_init sets the second kernel's
+// shared-memory limit for these dimensions (once per handle).
+cudaError_t final_init(const StepDims& d);
+void launch_final_norm(const StepDims& d, float* h, const float* part, int n_parts,
+                       long long part_stride, const float* mod, float* yF, cudaStream_t s);
+void launch_velocity_euler(const StepDims& d, const float* yF, const float* w_out_t,
+                           const float* b_out, const float* dt, float* buffer, float* out_chunk,
+                           float* vel_out, const float* fresh, unsigned long long seed,
+                           const unsigned long long* step_idx, cudaStream_t s);
+
+// out = silu(in W^T + bias), bf16 [M, K] x [N, K] -> bf16 [M, N]; K a multiple of 8.
+// gemv_init sets the shared-memory limit for K (once per handle).
+cudaError_t gemv_init(int K);
+void launch_gemv_silu(const void* in, const void* w, const float* bias, void* out, int M, int N,
+                      int K, cudaStream_t s);
 
 void launch_rope_table(float2* table, int n_pos, int dh, float theta, cudaStream_t s);
 
@@ -127,7 +144,9 @@ constexpr int kAttnKeysPerSplit = 256;
 constexpr int kAttnKeyBlock = 64;
 
 cudaError_t tc_attention_init();
-// Attention kernel, then (when a tile can have several key splits) the merge kernel.
+// Attention kernel; launch_attn_merge then combines the key splits (it launches
+// nothing when no tile can have more than one split).
+cudaError_t launch_attn_merge(const AttnArgs& a, int B, cudaStream_t s);
 cudaError_t launch_tc_attention(const CUtensorMap* q, const CUtensorMap* k,
                                 const CUtensorMap* v, const AttnArgs& a, int B,
                                 cudaStream_t s);

@@ -10,35 +10,46 @@ namespace fva {
 // ----------------------------------------------------------------------------
 // sinusoidal timestep embedding of every chunk's noise level (App. A.4 FiLM
 // condition input): e = [sin(2 pi tau / p_j) | cos(2 pi tau / p_j)],
-// p_j = t_min (t_max / t_min)^(j / (W/2 - 1)).  Arguments in double precision.
+// p_j = t_min (t_max / t_min)^(j / (W/2 - 1)).
+// The argument in half turns, x = tau * (2 / p_j), is formed from a two-float
+// split c_hi + c_lo of 2 / p_j (computed in double on the host): the product
+// tau * c_hi is split exactly with an fma, its integer part is removed exactly,
+// and sincospi of the small remainder gives sin / cos to fp32 accuracy.
 // ----------------------------------------------------------------------------
 template <typename Act>
-__global__ void temb_kernel(const float* __restrict__ tau, int W, double tmin, double tmax,
-                            Act* __restrict__ out) {
-  const int row = blockIdx.x;
+__global__ void temb_kernel(const float* __restrict__ tau, const float2* __restrict__ freq,
+                            int W, Act* __restrict__ out) {
+  const int row = blockIdx.y;
   const int half = W / 2;
   pdl_trigger();
   pdl_wait();
-  const double t = (double)tau[row];
-  for (int j = threadIdx.x; j < half; j += blockDim.x) {
-    const double period = tmin * pow(tmax / tmin, (double)j / (double)(half - 1));
-    const double arg = 2.0 * 3.14159265358979323846 * t / period;
-    double sn, cs;
-    sincos(arg, &sn, &cs);
-    out[(size_t)row * W + j] = from_float<Act>((float)sn);
-    out[(size_t)row * W + half + j] = from_float<Act>((float)cs);
+  const float t = tau[row];
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= half) return;
+  const float2 c = freq[j];
+  const float p = t * c.x;
+  const float p_err = fmaf(t, c.x, -p);      // exact remainder of the product
+  const float n = rintf(p);                  // |p| < 2^23: exact
+  const float r = (p - n) + fmaf(t, c.y, p_err);
+  float sn, cs;
+  sincospif(r, &sn, &cs);
+  const int odd = ((int)n) & 1;              // sin / cos of (n + r) pi
+  if (odd) {
+    sn = -sn;
+    cs = -cs;
   }
+  out[(size_t)row * W + j] = from_float<Act>(sn);
+  out[(size_t)row * W + half + j] = from_float<Act>(cs);
 }
 
-void launch_temb(const float* tau, int rows, int W, float tmin, float tmax, void* out,
+void launch_temb(const float* tau, const float2* freq, int rows, int W, void* out,
                  bool act_bf16, cudaStream_t s) {
   if (rows <= 0) return;
+  dim3 grid((W / 2 + 127) / 128, rows);
   if (act_bf16)
-    launch_pdl(temb_kernel<bf16>, dim3(rows), dim3(256), 0, s, tau, W, (double)tmin,
-               (double)tmax, (bf16*)out);
+    launch_pdl(temb_kernel<bf16>, grid, dim3(128), 0, s, tau, freq, W, (bf16*)out);
   else
-    launch_pdl(temb_kernel<float>, dim3(rows), dim3(256), 0, s, tau, W, (double)tmin,
-               (double)tmax, (float*)out);
+    launch_pdl(temb_kernel<float>, grid, dim3(128), 0, s, tau, freq, W, (float*)out);
 }
 
 // ----------------------------------------------------------------------------
@@ -102,12 +113,14 @@ template <typename Act>
 __global__ void embed_norm_kernel(StepDims d, const float* __restrict__ buffer,
                                   const float* __restrict__ w_in_t,
                                   const float* __restrict__ b_in, const float* __restrict__ mod,
-                                  float* __restrict__ h, Act* __restrict__ y) {
+                                  float* __restrict__ h, Act* __restrict__ y,
+                                  const L2Prefetch pf) {
   __shared__ float xs[128];
   __shared__ float red[32];
   const int m = blockIdx.x;
   const int r = m / d.T, t = m % d.T, c = t / d.H;
   pdl_trigger();
+  issue_l2_prefetch(pf);
   pdl_wait();
   const float* x = buffer + (size_t)m * d.A;  // buffer [B, K, H, A] = rows of A
   for (int a = threadIdx.x; a < d.A; a += blockDim.x) xs[a] = x[a];
@@ -135,15 +148,16 @@ __global__ void embed_norm_kernel(StepDims d, const float* __restrict__ buffer,
 
 void launch_embed_norm(const StepDims& d, const float* buffer, const float* w_in_t,
                        const float* b_in, const float* mod, float* h, void* y, bool act_bf16,
-                       cudaStream_t s) {
+                       const L2Prefetch* pf, cudaStream_t s) {
   const int rows = d.B * d.T;
   if (rows <= 0) return;
+  const L2Prefetch none = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
   if (act_bf16)
     launch_pdl(embed_norm_kernel<bf16>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, buffer,
-               w_in_t, b_in, mod, h, (bf16*)y);
+               w_in_t, b_in, mod, h, (bf16*)y, pf ? *pf : none);
   else
     launch_pdl(embed_norm_kernel<float>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, buffer,
-               w_in_t, b_in, mod, h, (float*)y);
+               w_in_t, b_in, mod, h, (float*)y, pf ? *pf : none);
 }
 
 // ----------------------------------------------------------------------------
@@ -155,11 +169,12 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
                                   const float* __restrict__ part, int n_parts,
                                   long long part_stride, const float* __restrict__ mod,
                                   int gate_off, int scale_off, int shift_off,
-                                  Act* __restrict__ y) {
+                                  Act* __restrict__ y, const L2Prefetch pf) {
   __shared__ float red[32];
   const int m = blockIdx.x;
   const int r = m / d.T, c = (m % d.T) / d.H;
   pdl_trigger();
+  issue_l2_prefetch(pf);
   pdl_wait();
   const float* mrow = mod + (size_t)(r * d.K + c) * d.N_mod;
   float* hrow = h + (size_t)m * d.W;
@@ -187,15 +202,19 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
 
 void launch_resid_norm(const StepDims& d, float* h, const float* part, int n_parts,
                        long long part_stride, const float* mod, int gate_off, int scale_off,
-                       int shift_off, void* y, bool act_bf16, cudaStream_t s) {
+                       int shift_off, void* y, bool act_bf16, const L2Prefetch* pf,
+                       cudaStream_t s) {
   const int rows = d.B * d.T;
   if (rows <= 0) return;
+  const L2Prefetch none = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
   if (act_bf16)
     launch_pdl(resid_norm_kernel<bf16>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h, part,
-               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (bf16*)y);
+               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (bf16*)y,
+               pf ? *pf : none);
   else
     launch_pdl(resid_norm_kernel<float>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h, part,
-               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (float*)y);
+               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (float*)y,
+               pf ? *pf : none);
 }
 
 // ----------------------------------------------------------------------------
@@ -233,106 +252,216 @@ __device__ __forceinline__ float tail_normal(unsigned long long seed, unsigned l
 }
 
 // ----------------------------------------------------------------------------
-// Final kernel.  One CTA per (token position j within a chunk, request r): it
-// owns column j of every chunk of request r, so the in-place roll of the buffer
-// is race-free.  For every chunk k: finish the residual stream, final FiLM
-// RMSNorm, velocity v = y W_out^T + b_out; then x'_k = x_k + dt_k v_k (fp32,
-// separately rounded multiply and add), out = x'_1, slot k <- x'_{k+1},
-// tail <- z.
+// Velocity, Euler update, emit, roll and tail.  The final FiLM RMSNorm has
+// already written y_F [B*K*H, W] (fp32).  One CTA per (token position j within
+// a chunk, request r) owns column j of every chunk of request r, so the
+// in-place roll of the buffer is race-free.  The K rows of y_F and (a slice of)
+// W_out^T [W, A] are staged in shared memory with all loads in flight at once;
+// thread (k, a) then computes v[k][a] = b_out[a] + sum_w y_F[k][w] W_out^T[w][a].
+// x'_k = x_k + dt_k v_k (fp32, separately rounded multiply and add), out = x'_1,
+// slot k <- x'_{k+1}, tail <- z.
 // ----------------------------------------------------------------------------
-__global__ void final_kernel(StepDims d, float* __restrict__ h, const float* __restrict__ part,
-                             int n_parts, long long part_stride, const float* __restrict__ mod,
-                             const float* __restrict__ w_out, const float* __restrict__ b_out,
-                             const float* __restrict__ dt, float* __restrict__ buffer,
-                             float* __restrict__ out_chunk, float* __restrict__ vel_out,
-                             const float* __restrict__ fresh, unsigned long long seed,
-                             const unsigned long long* __restrict__ step_idx) {
-  extern __shared__ float vs[];  // [K, A] velocities of this column
+constexpr int kVelThreads = 512;
+
+__global__ void __launch_bounds__(kVelThreads)
+    velocity_euler_kernel(StepDims d, const float* __restrict__ yF,
+                          const float* __restrict__ w_out_t, const float* __restrict__ b_out,
+                          const float* __restrict__ dt, float* __restrict__ buffer,
+                          float* __restrict__ out_chunk, float* __restrict__ vel_out,
+                          const float* __restrict__ fresh, unsigned long long seed,
+                          const unsigned long long* __restrict__ step_idx, int wchunk) {
+  extern __shared__ __align__(16) float sm[];
+  __shared__ __align__(8) uint64_t bar;
   const int j = blockIdx.x, r = blockIdx.y;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-  const int lgate = mod_off(d.L - 1, 5, d.W);
+  const int KA = d.K * d.A;
+  float* ys = sm;                    // [K][wchunk]
+  float* ws = ys + d.K * wchunk;     // [wchunk][A]
+  float* xs = ws + wchunk * d.A;     // [K][A] buffer values of this column
+  float* vs = xs + KA;               // [K][A] velocities
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
   pdl_trigger();
   pdl_wait();
-  for (int k = warp; k < d.K; k += nw) {
-    const int t = k * d.H + j;
-    const size_t m = (size_t)r * d.T + t;
-    const float* mrow = mod + (size_t)(r * d.K + k) * d.N_mod;
-    float* hrow = h + m * d.W;
-    float ss = 0.f;
-    for (int col = lane * 4; col < d.W; col += 128) {
-      float4 acc = __ldcg(reinterpret_cast<const float4*>(part + m * d.W + col));
-      for (int z = 1; z < n_parts; ++z) {
-        const float4 p =
-            __ldcg(reinterpret_cast<const float4*>(part + z * part_stride + m * d.W + col));
-        acc.x += p.x; acc.y += p.y; acc.z += p.z; acc.w += p.w;
+  const size_t slot = (size_t)d.H * d.A;
+  const float* xcol = buffer + ((size_t)r * d.K * d.H + j) * d.A;  // + k*slot selects chunk k
+  for (int i = threadIdx.x; i < KA; i += blockDim.x) {
+    xs[i] = xcol[(i / d.A) * slot + i % d.A];
+    vs[i] = b_out[i % d.A];
+  }
+  uint32_t phase = 0;
+  for (int w0 = 0; w0 < d.W; w0 += wchunk) {
+    __syncthreads();  // previous chunk consumed
+    if (threadIdx.x == 0) {
+      // all staging as bulk copies in flight at once: K rows of y_F and the W_out^T slice
+      mbar_arrive_expect_tx(&bar, (uint32_t)(sizeof(float) * (d.K + d.A) * wchunk));
+      for (int k = 0; k < d.K; ++k) {
+        const size_t m = (size_t)r * d.T + (size_t)k * d.H + j;
+        bulk_load(ys + k * wchunk, yF + m * d.W + w0, sizeof(float) * wchunk, &bar);
       }
-      const float4 g = *reinterpret_cast<const float4*>(mrow + lgate + col);
-      float4 hv = *reinterpret_cast<const float4*>(hrow + col);
-      hv.x = fmaf(g.x, acc.x, hv.x);
-      hv.y = fmaf(g.y, acc.y, hv.y);
-      hv.z = fmaf(g.z, acc.z, hv.z);
-      hv.w = fmaf(g.w, acc.w, hv.w);
-      *reinterpret_cast<float4*>(hrow + col) = hv;
-      ss += hv.x * hv.x + hv.y * hv.y + hv.z * hv.z + hv.w * hv.w;
+      bulk_load(ws, w_out_t + (size_t)w0 * d.A, (uint32_t)(sizeof(float) * wchunk * d.A), &bar);
     }
-    ss = warp_sum(ss);
-    const float rn = rsqrtf(ss / (float)d.W + d.eps);
-    const float* sF = mrow + modf_off(d.L, 0, d.W);
-    const float* bF = mrow + modf_off(d.L, 1, d.W);
-    for (int a0 = 0; a0 < d.A; a0 += 32) {
-      float acc[32];
-#pragma unroll
-      for (int i = 0; i < 32; ++i) acc[i] = 0.f;
-      for (int col = lane * 4; col < d.W; col += 128) {
-        const float4 hv = *reinterpret_cast<const float4*>(hrow + col);
-        const float4 sc = *reinterpret_cast<const float4*>(sF + col);
-        const float4 sh = *reinterpret_cast<const float4*>(bF + col);
-        const float y0 = hv.x * rn * (1.f + sc.x) + sh.x, y1 = hv.y * rn * (1.f + sc.y) + sh.y;
-        const float y2 = hv.z * rn * (1.f + sc.z) + sh.z, y3 = hv.w * rn * (1.f + sc.w) + sh.w;
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          if (a0 + i < d.A) {
-            const float4 w = *reinterpret_cast<const float4*>(w_out + (size_t)(a0 + i) * d.W + col);
-            acc[i] = fmaf(y0, w.x, fmaf(y1, w.y, fmaf(y2, w.z, fmaf(y3, w.w, acc[i]))));
-          }
-        }
+    mbar_wait(&bar, phase, nullptr, 0);
+    phase ^= 1u;
+    for (int i = threadIdx.x; i < KA; i += blockDim.x) {
+      const int k = i / d.A, a = i % d.A;
+      const float* yk = ys + k * wchunk;
+      float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
+      for (int w = 0; w < wchunk; w += 4) {
+        acc0 = fmaf(yk[w], ws[w * d.A + a], acc0);
+        acc1 = fmaf(yk[w + 1], ws[(w + 1) * d.A + a], acc1);
+        acc2 = fmaf(yk[w + 2], ws[(w + 2) * d.A + a], acc2);
+        acc3 = fmaf(yk[w + 3], ws[(w + 3) * d.A + a], acc3);
       }
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        const float s = warp_sum(acc[i]);
-        if (lane == i && a0 + i < d.A) vs[k * d.A + a0 + i] = s + b_out[a0 + i];
-      }
+      vs[i] += (acc0 + acc1) + (acc2 + acc3);
     }
   }
   __syncthreads();
   const unsigned long long step = *step_idx;
   const float* dtr = dt + (size_t)r * d.K;
+  float* colw = buffer + ((size_t)r * d.K * d.H + j) * d.A;
+  for (int i = threadIdx.x; i < KA; i += blockDim.x) {
+    const int k = i / d.A, a = i % d.A;
+    const float v = vs[i];
+    const float xk = __fadd_rn(xs[i], __fmul_rn(dtr[k], v));
+    if (k == 0)
+      out_chunk[((size_t)r * d.H + j) * d.A + a] = xk;
+    else
+      colw[(size_t)(k - 1) * slot + a] = xk;
+    if (vel_out) vel_out[(((size_t)r * d.K + k) * d.H + j) * d.A + a] = v;
+  }
   for (int a = threadIdx.x; a < d.A; a += blockDim.x) {
-    float* col = buffer + ((size_t)r * d.K * d.H + j) * d.A + a;  // + k*H*A selects the slot
-    const size_t slot = (size_t)d.H * d.A;
-    out_chunk[((size_t)r * d.H + j) * d.A + a] = __fadd_rn(col[0], __fmul_rn(dtr[0], vs[a]));
-    if (vel_out) vel_out[((size_t)r * d.K * d.H + j) * d.A + a] = vs[a];
-    for (int k = 1; k < d.K; ++k) {
-      const float v = vs[k * d.A + a];
-      const float xk = __fadd_rn(col[k * slot], __fmul_rn(dtr[k], v));
-      col[(k - 1) * slot] = xk;
-      if (vel_out) vel_out[(((size_t)r * d.K + k) * d.H + j) * d.A + a] = v;
-    }
     const int e = j * d.A + a;
-    col[(size_t)(d.K - 1) * slot] =
+    colw[(size_t)(d.K - 1) * slot + a] =
         fresh ? fresh[(size_t)r * d.H * d.A + e] : tail_normal(seed, step, r, e);
   }
 }
 
-void launch_final(const StepDims& d, float* h, const float* part, int n_parts,
-                  long long part_stride, const float* mod, const float* w_out,
-                  const float* b_out, const float* dt, float* buffer, float* out_chunk,
-                  float* vel_out, const float* fresh, unsigned long long seed,
-                  const unsigned long long* step_idx, cudaStream_t s) {
-  dim3 grid(d.H, d.B);
-  const size_t smem = sizeof(float) * d.K * d.A;
-  launch_pdl(final_kernel, grid, dim3(256), smem, s, d, h, part, n_parts, part_stride, mod,
-             w_out, b_out, dt, buffer, out_chunk, vel_out, fresh, seed, step_idx);
+// Largest W-chunk (a divisor of W, multiple of 4) whose staging fits ~200 KB.
+// Every bulk copy then starts 16-byte aligned (W and the chunk are multiples of 4).
+static int vel_chunk(const StepDims& d) {
+  const size_t budget = 200 * 1024 - sizeof(float) * 2 * d.K * d.A;
+  int c = d.W;
+  while (c > 4 && (sizeof(float) * (size_t)(d.K + d.A) * c > budget || d.W % c || c % 4)) --c;
+  return c;
+}
+
+static size_t vel_smem_bytes(const StepDims& d) {
+  return sizeof(float) * ((size_t)2 * d.K * d.A + (size_t)(d.K + d.A) * vel_chunk(d));
+}
+
+cudaError_t final_init(const StepDims& d) {
+  return cudaFuncSetAttribute(velocity_euler_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)vel_smem_bytes(d));
+}
+
+void launch_final_norm(const StepDims& d, float* h, const float* part, int n_parts,
+                       long long part_stride, const float* mod, float* yF, cudaStream_t s) {
+  launch_resid_norm(d, h, part, n_parts, part_stride, mod, mod_off(d.L - 1, 5, d.W),
+                    modf_off(d.L, 0, d.W), modf_off(d.L, 1, d.W), yF, false, nullptr, s);
+}
+
+void launch_velocity_euler(const StepDims& d, const float* yF, const float* w_out_t,
+                           const float* b_out, const float* dt, float* buffer, float* out_chunk,
+                           float* vel_out, const float* fresh, unsigned long long seed,
+                           const unsigned long long* step_idx, cudaStream_t s) {
+  launch_pdl(velocity_euler_kernel, dim3(d.H, d.B), dim3(kVelThreads), vel_smem_bytes(d), s, d,
+             yF, w_out_t, b_out, dt, buffer, out_chunk, vel_out, fresh, seed, step_idx,
+             vel_chunk(d));
+}
+
+// ----------------------------------------------------------------------------
+// Time MLP layer (App. A.4 condition): out = silu(in W^T + b) for the few rows
+// M = B*K of per-chunk timestep features; bf16 in / weights / out, fp32 math.
+// One warp per output column; each CTA stages 16 input rows in shared memory and
+// each lane reads 8 contiguous weights per 16-byte load.  K a multiple of 8.
+// ----------------------------------------------------------------------------
+constexpr int kGemvRows = 16;
+constexpr int kGemvWarps = 8;
+constexpr int kGemvMaxK8 = 512;  // K <= 4096: each lane keeps its weights in registers
+
+__global__ void __launch_bounds__(32 * kGemvWarps)
+    gemv_silu_kernel(const bf16* __restrict__ in, const bf16* __restrict__ w,
+                     const float* __restrict__ bias, bf16* __restrict__ out, int M, int N,
+                     int K) {
+  extern __shared__ __align__(16) uint4 sin4[];  // [16][K/8]
+  __shared__ __align__(8) uint64_t bar;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n = blockIdx.x * kGemvWarps + warp;
+  const int k8 = K / 8;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
+  // this warp's weight row: lane holds chunks lane, lane+32, ... (weights do not
+  // depend on earlier kernels, so they are requested before waiting)
+  uint4 wv[kGemvMaxK8 / 32];
+  const uint4* wr = reinterpret_cast<const uint4*>(w + (size_t)min(n, N - 1) * K);
+#pragma unroll
+  for (int i = 0; i < kGemvMaxK8 / 32; ++i)
+    if (lane + 32 * i < k8) wv[i] = __ldg(wr + lane + 32 * i);
+  pdl_trigger();
+  pdl_wait();
+  uint32_t phase = 0;
+  for (int m0 = 0; m0 < M; m0 += kGemvRows) {
+    const int mr = min(kGemvRows, M - m0);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      mbar_arrive_expect_tx(&bar, (uint32_t)(mr * K * 2));
+      bulk_load(sin4, in + (size_t)m0 * K, (uint32_t)(mr * K * 2), &bar);
+    }
+    mbar_wait(&bar, phase, nullptr, 0);
+    phase ^= 1u;
+    float acc[kGemvRows];
+#pragma unroll
+    for (int mm = 0; mm < kGemvRows; ++mm) acc[mm] = 0.f;
+#pragma unroll
+    for (int i = 0; i < kGemvMaxK8 / 32; ++i) {
+      const int c = lane + 32 * i;
+      if (c >= k8) break;
+      const __nv_bfloat162* w2 = reinterpret_cast<const __nv_bfloat162*>(&wv[i]);
+      float wf[8];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float2 f = __bfloat1622float2(w2[u]);
+        wf[2 * u] = f.x;
+        wf[2 * u + 1] = f.y;
+      }
+#pragma unroll
+      for (int mm = 0; mm < kGemvRows; ++mm) {
+        if (mm >= mr) break;
+        const uint4 xv = sin4[mm * k8 + c];
+        const __nv_bfloat162* x2 = reinterpret_cast<const __nv_bfloat162*>(&xv);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const float2 f = __bfloat1622float2(x2[u]);
+          acc[mm] = fmaf(f.x, wf[2 * u], fmaf(f.y, wf[2 * u + 1], acc[mm]));
+        }
+      }
+    }
+#pragma unroll
+    for (int mm = 0; mm < kGemvRows; ++mm) {
+      const float v = warp_sum(acc[mm]);
+      if (lane == mm && mm < mr && n < N)
+        out[(size_t)(m0 + mm) * N + n] = __float2bfloat16_rn(silu_f(v + bias[n]));
+    }
+  }
+}
+
+cudaError_t gemv_init(int K) {
+  return cudaFuncSetAttribute(gemv_silu_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              kGemvRows * K * 2);
+}
+
+void launch_gemv_silu(const void* in, const void* w, const float* bias, void* out, int M, int N,
+                      int K, cudaStream_t s) {
+  if (M <= 0) return;
+  launch_pdl(gemv_silu_kernel, dim3((N + kGemvWarps - 1) / kGemvWarps), dim3(32 * kGemvWarps),
+             (size_t)kGemvRows * K * 2, s, (const bf16*)in, (const bf16*)w, bias, (bf16*)out, M, N,
+             K);
 }
 
 // ----------------------------------------------------------------------------

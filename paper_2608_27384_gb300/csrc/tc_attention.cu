@@ -10,14 +10,15 @@
 // tile in shared memory serves every head.  The key range of a tile is cut into
 // splits of 256 keys (4 blocks of 64); key blocks past the tile's largest limit
 // are never loaded.  One CTA handles one (tile, split):
-//   warp 0      TMA: Q tile (64 KB, loaded once) then K blocks, then V blocks,
-//               through a 2-slot ring of 32 KB;
+//   warp 0      TMA: the Q tile (64 KB) and all K blocks at once, then the V
+//               blocks as K slots free up (4-slot ring of 32 KB);
 //   warp 1      TMEM (512 columns: S in 0..255, O in 256..511); one lane issues
 //               S = Q K^T per key block (M=128, N=64, K=16 steps over dh), and,
 //               after the softmax, O = P V (M=128, N=256, MN-major V);
-//   warps 2..5  one thread per query row: exact row max over the split's visible
-//               keys, P = exp(S - max) written as bf16 into the swizzled A-operand
-//               layout in shared memory, row sum; then read O from TMEM.
+//   warps 2..17 softmax + epilogue, four threads per query row (one per
+//               64-key block / 64 head-dim columns): exact row max over the
+//               split's visible keys, P = exp(S - max) written as bf16 over the Q
+//               tile (Q is dead once S is complete), row sum; then O from TMEM.
 // A tile with one split writes O / l as bf16.  Otherwise each split writes its
 // unnormalised (O, max, sum) to scratch and attn_merge_kernel combines the
 // splits of every row in split order (deterministic) and writes bf16.
@@ -30,15 +31,20 @@ namespace {
 
 constexpr int kDH = 256;
 constexpr int kRows = 128;
-constexpr int kKB = kAttnKeyBlock;                    // 64 keys per block
+constexpr int kKB = kAttnKeyBlock;                        // 64 keys per block
 constexpr int kBlocksPerSplit = kAttnKeysPerSplit / kKB;  // 4
-constexpr int kQBytes = kRows * kDH * 2;              // 64 KB
-constexpr int kPBytes = kRows * kAttnKeysPerSplit * 2;  // 64 KB
-constexpr int kKVBytes = kKB * kDH * 2;               // 32 KB per K or V block
-constexpr int kSlots = 2;
-constexpr int kSmem = kQBytes + kPBytes + kSlots * kKVBytes + 1024 + 256;
-constexpr int kThreads = 192;
+constexpr int kQBytes = kRows * kDH * 2;                  // 64 KB (Q, later P)
+constexpr int kKVBytes = kKB * kDH * 2;                   // 32 KB per K or V block
+constexpr int kSlots = 4;
+constexpr int kSoftmaxThreads = 512;
+constexpr int kThreads = 64 + kSoftmaxThreads;
+constexpr int kSmem = kQBytes + kSlots * kKVBytes + 1024 /*align*/ + 1024 /*bars*/ +
+                      8 * kRows * 4 /*row exchange*/;
 constexpr uint32_t kTmemCols = 512;
+
+__device__ __forceinline__ void softmax_bar() {
+  asm volatile("bar.sync 1, 512;" ::: "memory");
+}
 
 __global__ void __launch_bounds__(kThreads, 1)
     tc_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
@@ -61,17 +67,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* sQ = smem;                       // 4 slabs [128 rows x 128 B]
-  uint8_t* sP = smem + kQBytes;             // 4 slabs [128 rows x 128 B]
-  uint8_t* sKV = sP + kPBytes;              // 2 slots x 4 slabs [64 rows x 128 B]
+  uint8_t* sQP = smem;                      // 4 slabs [128 rows x 128 B]: Q, then P
+  uint8_t* sKV = smem + kQBytes;            // 4 slots x 4 slabs [64 rows x 128 B]
   uint64_t* bars = (uint64_t*)(sKV + kSlots * kKVBytes);
   uint64_t* q_full = bars + 0;
-  uint64_t* kv_full = bars + 1;   // [2]
-  uint64_t* kv_empty = bars + 3;  // [2]
-  uint64_t* s_full = bars + 5;
-  uint64_t* p_full = bars + 6;
-  uint64_t* o_full = bars + 7;
-  uint32_t* tmem_slot = (uint32_t*)(bars + 8);
+  uint64_t* kv_full = bars + 1;   // [4]
+  uint64_t* kv_empty = bars + 5;  // [4]
+  uint64_t* s_full = bars + 9;
+  uint64_t* p_full = bars + 10;
+  uint64_t* o_full = bars + 11;
+  uint32_t* tmem_slot = (uint32_t*)(bars + 12);
+  float* xmax = (float*)(bars + 128);   // [4][128] per-block row max
+  float* xsum = xmax + 4 * kRows;       // [4][128] per-block row sum
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -81,7 +88,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&kv_empty[s], 1);
     }
     mbar_init(s_full, 1);
-    mbar_init(p_full, kRows);
+    mbar_init(p_full, kSoftmaxThreads);
     mbar_init(o_full, 1);
     fence_barrier_init();
     tma_prefetch_desc(&tmQ);
@@ -95,20 +102,31 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  pdl_trigger();
-  pdl_wait();  // q and the action K/V come from the QKV projection
   const uint32_t tS = tmem, tO = tmem + 256;
+  pdl_trigger();
 
   const int qrow0 = (r * a.T + t0) * a.nq;
   const int krow0 = a.kv_row0 + r * a.S_cap + kb0 * kKB;
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer
+    // Key blocks that lie wholly inside the prefix come from fva_set_prefix_kv,
+    // not from the predecessor grid, so they are requested before waiting for
+    // it; q and the action keys/values (written by the QKV projection) after.
+    // Every other thread only runs behind these loads.
+    int it = 0;
+    for (; it < nblk && (kb0 + it + 1) * kKB <= P; ++it) {  // first use of slot it
+      mbar_arrive_expect_tx(&kv_full[it], kKVBytes);
+      for (int j = 0; j < 4; ++j)
+        tma_load_2d(sKV + it * kKVBytes + j * (kKB * 128), &tmK, j * 64, krow0 + it * kKB,
+                    &kv_full[it]);
+    }
+    pdl_wait();
     mbar_arrive_expect_tx(q_full, kQBytes);
-    for (int j = 0; j < 4; ++j) tma_load_2d(sQ + j * (kRows * 128), &tmQ, j * 64, qrow0, q_full);
-    for (int it = 0; it < 2 * nblk; ++it) {
-      const int s = it & 1;
-      const uint32_t ph = (uint32_t)(it >> 1) & 1u;
+    for (int j = 0; j < 4; ++j) tma_load_2d(sQP + j * (kRows * 128), &tmQ, j * 64, qrow0, q_full);
+    for (; it < 2 * nblk; ++it) {
+      const int s = it % kSlots;
+      const uint32_t ph = (uint32_t)(it / kSlots) & 1u;
       if (!mbar_wait(&kv_empty[s], ph ^ 1u, a.err, KERR_WAIT_MMA)) break;
       const bool is_k = it < nblk;
       const int row = krow0 + (is_k ? it : it - nblk) * kKB;
@@ -123,10 +141,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t idesc_o = umma_idesc_bf16(kRows, kDH, true);
     bool good = mbar_wait(q_full, 0, a.err, KERR_WAIT_TMA);
     tc_fence_after();
-    const uint32_t q_base = smem_u32(sQ), p_base = smem_u32(sP), kv_base = smem_u32(sKV);
+    const uint32_t qp_base = smem_u32(sQP), kv_base = smem_u32(sKV);
     for (int it = 0; good && it < nblk; ++it) {
-      const int s = it & 1;
-      if (!mbar_wait(&kv_full[s], (uint32_t)(it >> 1) & 1u, a.err, KERR_WAIT_TMA)) {
+      const int s = it % kSlots;
+      if (!mbar_wait(&kv_full[s], (uint32_t)(it / kSlots) & 1u, a.err, KERR_WAIT_TMA)) {
         good = false;
         break;
       }
@@ -135,7 +153,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int ks = 0; ks < kDH / 16; ++ks) {
         const uint32_t off = (ks & 3) * 32;  // 16 bf16 along K inside the 128-byte row
-        const uint64_t ad = umma_desc_sw128(q_base + (ks >> 2) * (kRows * 128) + off, 16, 1024);
+        const uint64_t ad = umma_desc_sw128(qp_base + (ks >> 2) * (kRows * 128) + off, 16, 1024);
         const uint64_t bd = umma_desc_sw128(kb + (ks >> 2) * (kKB * 128) + off, 16, 1024);
         umma_bf16(tS + it * kKB, ad, bd, idesc_s, ks > 0 ? 1u : 0u);
       }
@@ -145,8 +163,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (good) good = mbar_wait(p_full, 0, a.err, KERR_WAIT_SYNC);
     tc_fence_after();
     for (int j = 0; good && j < nblk; ++j) {
-      const int it = nblk + j, s = it & 1;
-      if (!mbar_wait(&kv_full[s], (uint32_t)(it >> 1) & 1u, a.err, KERR_WAIT_TMA)) {
+      const int it = nblk + j, s = it % kSlots;
+      if (!mbar_wait(&kv_full[s], (uint32_t)(it / kSlots) & 1u, a.err, KERR_WAIT_TMA)) {
         good = false;
         break;
       }
@@ -154,7 +172,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t vb = kv_base + s * kKVBytes;
 #pragma unroll
       for (int ks = 0; ks < kKB / 16; ++ks) {
-        const uint64_t ad = umma_desc_sw128(p_base + j * (kRows * 128) + ks * 32, 16, 1024);
+        const uint64_t ad = umma_desc_sw128(qp_base + j * (kRows * 128) + ks * 32, 16, 1024);
         // V block [64 keys][256 dh] as 4 slabs of 64 dh: MN-major B operand.
         const uint64_t bd = umma_desc_sw128(vb + ks * 16 * 128, kKB * 128, 1024);
         umma_bf16(tO, ad, bd, idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
@@ -163,83 +181,96 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (good) umma_commit(o_full);
   } else if (warp >= 2) {
-    // ---------------- softmax + epilogue, one query row per thread
+    // ---------------- softmax + epilogue: thread (key block g, row)
+    const int g = (warp - 2) >> 2;          // key block of S / 64 dh columns of O
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;
     const int t = t0 + row / a.nq;
     const bool valid = t < a.T;
     const int limit = valid ? attn_key_limit(P, t, a.H) : 0;
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+    const bool has_blk = g < nblk;
+    const int key0 = (kb0 + g) * kKB;
     bool good = __all_sync(0xffffffffu, mbar_wait(s_full, 0, a.err, KERR_WAIT_MMA));
     tc_fence_after();
     float mx = -INFINITY, l = 0.f;
-    if (good) {
-      for (int j = 0; j < nblk; ++j) {
-        for (int hh = 0; hh < 2; ++hh) {
-          float v[32];
-          tmem_ld32(tS + lane_off + j * kKB + hh * 32, v);
-          const int key0 = (kb0 + j) * kKB + hh * 32;
+    uint32_t sv[64];
+    if (good && has_blk) {
+      uint32_t (&s0)[32] = *reinterpret_cast<uint32_t(*)[32]>(&sv[0]);
+      uint32_t (&s1)[32] = *reinterpret_cast<uint32_t(*)[32]>(&sv[32]);
+      tmem_ld32_nowait(tS + lane_off + g * kKB, s0);
+      tmem_ld32_nowait(tS + lane_off + g * kKB + 32, s1);
+      tmem_ld_wait();
+      if (key0 + kKB <= limit) {  // whole block visible
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (key0 + i < limit) mx = fmaxf(mx, v[i]);
-        }
-      }
-      const float mscaled = mx * a.scale_log2;
-      for (int j = 0; j < nblk; ++j) {
-        uint8_t* prow = sP + j * (kRows * 128) + row * 128;
-        for (int hh = 0; hh < 2; ++hh) {
-          float v[32];
-          tmem_ld32(tS + lane_off + j * kKB + hh * 32, v);
-          const int key0 = (kb0 + j) * kKB + hh * 32;
+        for (int i = 0; i < 64; ++i) mx = fmaxf(mx, __uint_as_float(sv[i]));
+      } else {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float p = (key0 + i < limit) ? exp2f(fmaf(v[i], a.scale_log2, -mscaled)) : 0.f;
-            const float pr = __bfloat162float(__float2bfloat16_rn(p));
-            l += pr;
-            v[i] = pr;
-          }
-#pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            const int chunk = hh * 4 + c;                       // 16-byte chunk in the row
-            const int phys = chunk ^ (row & 7);                 // 128-byte swizzle
-            *reinterpret_cast<uint4*>(prow + phys * 16) = pack_bf16x8(&v[c * 8]);
-          }
-        }
+        for (int i = 0; i < 64; ++i)
+          if (key0 + i < limit) mx = fmaxf(mx, __uint_as_float(sv[i]));
       }
     }
+    xmax[g * kRows + row] = mx;
+    softmax_bar();
+    mx = fmaxf(fmaxf(xmax[row], xmax[kRows + row]), fmaxf(xmax[2 * kRows + row], xmax[3 * kRows + row]));
+    if (good && has_blk) {
+      const float mscaled = mx * a.scale_log2;
+      uint8_t* prow = sQP + g * (kRows * 128) + row * 128;
+      const int nvis = min(kKB, max(0, limit - key0));
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {  // 16-byte chunk c = keys 8c .. 8c+7
+        float p[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int kk = c * 8 + i;
+          const float e = exp2f(fmaf(__uint_as_float(sv[kk]), a.scale_log2, -mscaled));
+          const float pr = kk < nvis ? __bfloat162float(__float2bfloat16_rn(e)) : 0.f;
+          l += pr;
+          p[i] = pr;
+        }
+        const int phys = c ^ (row & 7);  // 128-byte swizzle
+        *reinterpret_cast<uint4*>(prow + phys * 16) = pack_bf16x8(p);
+      }
+    }
+    xsum[g * kRows + row] = l;
     fence_proxy_async_smem();
     mbar_arrive(p_full);
     if (good) good = __all_sync(0xffffffffu, mbar_wait(o_full, 0, a.err, KERR_WAIT_MMA));
     tc_fence_after();
+    softmax_bar();  // xsum complete
+    l = (xsum[row] + xsum[kRows + row]) + (xsum[2 * kRows + row] + xsum[3 * kRows + row]);
     const int gtile = r * a.tiles_per_req + tile;
     const int grow = qrow0 + row;  // global q row = (r*T + t) * nq + head
+    const int c0 = g * 64;         // O columns of this thread
     if (good) {
-      if (nsplit == 1) {
-        const float inv = l > 0.f ? 1.f / l : 0.f;
-        for (int c = 0; c < kDH; c += 32) {
-          float v[32];
-          tmem_ld32(tO + lane_off + c, v);
-          if (!valid) continue;
+      uint32_t ov[64];
+      uint32_t (&o0)[32] = *reinterpret_cast<uint32_t(*)[32]>(&ov[0]);
+      uint32_t (&o1)[32] = *reinterpret_cast<uint32_t(*)[32]>(&ov[32]);
+      tmem_ld32_nowait(tO + lane_off + c0, o0);
+      tmem_ld32_nowait(tO + lane_off + c0 + 32, o1);
+      tmem_ld_wait();
+      if (valid) {
+        if (nsplit == 1) {
+          const float inv = l > 0.f ? 1.f / l : 0.f;
+          bf16* dst = (bf16*)a.out + (size_t)grow * kDH + c0;
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] *= inv;
-          bf16* dst = (bf16*)a.out + (size_t)grow * kDH + c;
+          for (int i = 0; i < 64; i += 8) {
+            float v[8];
 #pragma unroll
-          for (int i = 0; i < 32; i += 8) *reinterpret_cast<uint4*>(dst + i) = pack_bf16x8(&v[i]);
+            for (int u = 0; u < 8; ++u) v[u] = __uint_as_float(ov[i + u]) * inv;
+            *reinterpret_cast<uint4*>(dst + i) = pack_bf16x8(v);
+          }
+        } else {
+          float* po = a.part_o + (((size_t)gtile * a.max_splits + split) * kRows + row) * kDH + c0;
+#pragma unroll
+          for (int i = 0; i < 64; i += 4)
+            __stcg(reinterpret_cast<float4*>(po + i),
+                   make_float4(__uint_as_float(ov[i]), __uint_as_float(ov[i + 1]),
+                               __uint_as_float(ov[i + 2]), __uint_as_float(ov[i + 3])));
+          if (g == 0)
+            __stcg(a.part_ml + ((size_t)gtile * a.max_splits + split) * kRows + row,
+                   make_float2(mx, l));
         }
-      } else {
-        float* po = a.part_o + (((size_t)gtile * a.max_splits + split) * kRows + row) * kDH;
-        for (int c = 0; c < kDH; c += 32) {
-          float v[32];
-          tmem_ld32(tO + lane_off + c, v);
-          if (!valid) continue;
-#pragma unroll
-          for (int i = 0; i < 32; i += 4)
-            __stcg(reinterpret_cast<float4*>(po + c + i),
-                   make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]));
-        }
-        if (valid)
-          __stcg(a.part_ml + ((size_t)gtile * a.max_splits + split) * kRows + row,
-                 make_float2(mx, l));
       }
     }
   }
@@ -277,15 +308,27 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
   const float w = ml.y > 0.f ? exp2f((ml.x - m_all) * a.scale_log2) : 0.f;
   const float inv = 1.f / warp_sum(w * ml.y);
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-  for (int s = 0; s < nsplit; ++s) {
-    const float ws = __shfl_sync(0xffffffffu, w, s);
-    const float* po = a.part_o + ((tbase + s) * kRows + row) * kDH + lane * 8;
-    const float4 x0 = __ldcg(reinterpret_cast<const float4*>(po));
-    const float4 x1 = __ldcg(reinterpret_cast<const float4*>(po + 4));
-    acc[0] = fmaf(ws, x0.x, acc[0]); acc[1] = fmaf(ws, x0.y, acc[1]);
-    acc[2] = fmaf(ws, x0.z, acc[2]); acc[3] = fmaf(ws, x0.w, acc[3]);
-    acc[4] = fmaf(ws, x1.x, acc[4]); acc[5] = fmaf(ws, x1.y, acc[5]);
-    acc[6] = fmaf(ws, x1.z, acc[6]); acc[7] = fmaf(ws, x1.w, acc[7]);
+  for (int s0 = 0; s0 < nsplit; s0 += 8) {  // up to 8 splits' loads in flight
+    float4 x[8][2];
+    float ws[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      ws[u] = __shfl_sync(0xffffffffu, w, (s0 + u) & 31);
+      if (s0 + u < nsplit) {
+        const float* po = a.part_o + ((tbase + s0 + u) * kRows + row) * kDH + lane * 8;
+        x[u][0] = __ldcg(reinterpret_cast<const float4*>(po));
+        x[u][1] = __ldcg(reinterpret_cast<const float4*>(po + 4));
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      if (s0 + u < nsplit) {
+        acc[0] = fmaf(ws[u], x[u][0].x, acc[0]); acc[1] = fmaf(ws[u], x[u][0].y, acc[1]);
+        acc[2] = fmaf(ws[u], x[u][0].z, acc[2]); acc[3] = fmaf(ws[u], x[u][0].w, acc[3]);
+        acc[4] = fmaf(ws[u], x[u][1].x, acc[4]); acc[5] = fmaf(ws[u], x[u][1].y, acc[5]);
+        acc[6] = fmaf(ws[u], x[u][1].z, acc[6]); acc[7] = fmaf(ws[u], x[u][1].w, acc[7]);
+      }
+    }
   }
 #pragma unroll
   for (int i = 0; i < 8; ++i) acc[i] *= inv;
@@ -303,9 +346,12 @@ cudaError_t launch_tc_attention(const CUtensorMap* q, const CUtensorMap* k,
                                 const CUtensorMap* v, const AttnArgs& a, int B,
                                 cudaStream_t s) {
   if (a.max_splits > 32) return cudaErrorInvalidValue;  // the merge holds one split per lane
-  cudaError_t e = launch_pdl(tc_attn_kernel, dim3(a.tiles_per_req, a.max_splits, B),
-                             dim3(kThreads), kSmem, s, *q, *k, *v, a);
-  if (e != cudaSuccess || a.max_splits == 1) return e;
+  return launch_pdl(tc_attn_kernel, dim3(a.tiles_per_req, a.max_splits, B), dim3(kThreads),
+                    kSmem, s, *q, *k, *v, a);
+}
+
+cudaError_t launch_attn_merge(const AttnArgs& a, int B, cudaStream_t s) {
+  if (a.max_splits == 1) return cudaSuccess;
   return launch_pdl(attn_merge_kernel, dim3(a.tiles_per_req, B, kRows / 8), dim3(256), 0, s, a);
 }
 

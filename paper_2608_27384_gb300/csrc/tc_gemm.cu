@@ -104,9 +104,15 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
     else
       dst = (bf16*)(seg == ep.nq ? ep.kc : ep.vc) + ((size_t)r * ep.S_cap + pos) * dh;
     const bool rotate = seg <= ep.nq;
-    const float2* rope = ep.rope + (size_t)pos * (dh / 2);
+    const float4* cs4 = reinterpret_cast<const float4*>(ep.rope + (size_t)pos * (dh / 2) +
+                                                        tj * half);  // (cos, sin) pairs
 #pragma unroll 1
     for (int c = 0; c < half; c += 32) {
+      float4 cs[16];
+      if (ok && rotate) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) cs[i] = __ldg(cs4 + c / 2 + i);
+      }
       float x1[32], x2[32];
       tmem_ld32(trow + c, x1);
       tmem_ld32(trow + half + c, x2);
@@ -114,11 +120,12 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
       const int d0 = tj * half + c;
       if (rotate) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float2 cs = __ldg(rope + d0 + i);
-          const float a = x1[i], b = x2[i];
-          x1[i] = a * cs.x - b * cs.y;
-          x2[i] = b * cs.x + a * cs.y;
+        for (int i = 0; i < 32; i += 2) {
+          const float a0 = x1[i], b0 = x2[i], a1 = x1[i + 1], b1 = x2[i + 1];
+          x1[i] = a0 * cs[i / 2].x - b0 * cs[i / 2].y;
+          x2[i] = b0 * cs[i / 2].x + a0 * cs[i / 2].y;
+          x1[i + 1] = a1 * cs[i / 2].z - b1 * cs[i / 2].w;
+          x2[i + 1] = b1 * cs[i / 2].z + a1 * cs[i / 2].w;
         }
       }
       store_bf16x32(dst + d0, x1);
@@ -162,11 +169,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   pdl_trigger();
-  pdl_wait();  // A (and the epilogue's destinations) belong to earlier kernels
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer
-    for (int i = 0; i < nkb; ++i) {
+    // The weights (B) do not depend on earlier kernels: the first ring stages of
+    // B are requested before waiting for the predecessor grid.  A (activations)
+    // and everything downstream of it come after the wait; the MMA and epilogue
+    // threads only run behind these loads, so they are ordered after it too.
+    const int pre = min(nkb, C::kStages);
+    for (int i = 0; i < pre; ++i) {
+      mbar_arrive_expect_tx(&full[i], C::kStageBytes);
+      tma_load_2d(smem + i * C::kStageBytes + C::kABytes, &tmB, (kb0 + i) * kBK, n0, &full[i]);
+    }
+    pdl_wait();
+    for (int i = 0; i < pre; ++i)
+      tma_load_2d(smem + i * C::kStageBytes, &tmA, (kb0 + i) * kBK, m0, &full[i]);
+    for (int i = pre; i < nkb; ++i) {
       const int s = i % C::kStages;
       const uint32_t ph = (uint32_t)(i / C::kStages) & 1u;
       if (!mbar_wait(&empty[s], ph ^ 1u, ep.err, KERR_WAIT_MMA)) break;
