@@ -305,6 +305,48 @@ __device__ __forceinline__ bf16 from_float<bf16>(float x) { return __float2bfloa
 __device__ __forceinline__ float to_float(float x) { return x; }
 __device__ __forceinline__ float to_float(bf16 x) { return __bfloat162float(x); }
 
+// Coalesced row stores for one warp.  The tcgen05.ld layout gives one output
+// row per thread; storing straight from registers scatters every warp store
+// over 32 cache lines.  Instead each lane puts its row's pieces into a
+// warp-private shared-memory stage (32 rows x kRowBytes, pitch kRowBytes + 16,
+// 16-byte aligned) with stage_put, then stage_flush writes the tile with
+// consecutive lanes storing consecutive 16-byte pieces of a row, so each
+// instruction writes whole 128-byte lines.  dst_row is the lane's row
+// destination (nullptr skips the row).
+template <int kRowBytes, int kN>
+__device__ __forceinline__ void stage_put(uint8_t* stage, int lane, int byte_off,
+                                          const uint4 (&data)[kN]) {
+  constexpr int kPitch = kRowBytes + 16;
+#pragma unroll
+  for (int c = 0; c < kN; ++c)
+    *reinterpret_cast<uint4*>(stage + lane * kPitch + byte_off + c * 16) = data[c];
+}
+
+template <int kRowBytes>
+__device__ __forceinline__ void stage_flush(uint8_t* stage, void* dst_row, int lane) {
+  constexpr int kPitch = kRowBytes + 16;
+  constexpr int kChunks = kRowBytes / 16;
+  __syncwarp();
+  const unsigned long long my = reinterpret_cast<unsigned long long>(dst_row);
+#pragma unroll 4
+  for (int i = 0; i < kChunks; ++i) {
+    const int f = i * 32 + lane;  // flat 16-byte piece of the tile
+    const int r = f / kChunks, c = f % kChunks;
+    const unsigned long long d = __shfl_sync(0xffffffffu, my, r);
+    if (d)
+      *reinterpret_cast<uint4*>(d + c * 16) =
+          *reinterpret_cast<const uint4*>(stage + r * kPitch + c * 16);
+  }
+  __syncwarp();
+}
+
+template <int kBytes>
+__device__ __forceinline__ void warp_store_rows(uint8_t* stage, const uint4 (&data)[kBytes / 16],
+                                                void* dst_row, int lane) {
+  stage_put<kBytes>(stage, lane, 0, data);
+  stage_flush<kBytes>(stage, dst_row, lane);
+}
+
 // 8 floats -> 8 bf16 packed in a uint4 (for 16-byte stores).
 __device__ __forceinline__ uint4 pack_bf16x8(const float* f) {
   uint4 u;

@@ -101,7 +101,7 @@ __device__ __forceinline__ void modulated_norm_row(const float* __restrict__ hro
 
 inline int row_threads(int W) {
   int t = W / 4;
-  t = t < 32 ? 32 : (t > 256 ? 256 : t);
+  t = t < 32 ? 32 : (t > 1024 ? 1024 : t);
   return (t + 31) & ~31;
 }
 
@@ -178,21 +178,55 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
   pdl_wait();
   const float* mrow = mod + (size_t)(r * d.K + c) * d.N_mod;
   float* hrow = h + (size_t)m * d.W;
-  float ss = 0.f;
-  for (int col = threadIdx.x * 4; col < d.W; col += blockDim.x * 4) {
-    float4 acc = __ldcg(reinterpret_cast<const float4*>(part + (size_t)m * d.W + col));
-    for (int z = 1; z < n_parts; ++z) {
-      const float4 p =
-          __ldcg(reinterpret_cast<const float4*>(part + z * part_stride + (size_t)m * d.W + col));
-      acc.x += p.x; acc.y += p.y; acc.z += p.z; acc.w += p.w;
-    }
+  const int col = threadIdx.x * 4;
+  if (d.W == 4 * (int)blockDim.x) {
+    // one float4 per thread: every load in flight at once, values kept in registers
+    float4 p[8];
+#pragma unroll
+    for (int z = 0; z < 8; ++z)
+      if (z < n_parts)
+        p[z] = __ldcg(reinterpret_cast<const float4*>(part + z * part_stride + (size_t)m * d.W + col));
     const float4 g = *reinterpret_cast<const float4*>(mrow + gate_off + col);
+    const float4 sc = *reinterpret_cast<const float4*>(mrow + scale_off + col);
+    const float4 sh = *reinterpret_cast<const float4*>(mrow + shift_off + col);
     float4 hv = *reinterpret_cast<const float4*>(hrow + col);
+    float4 acc = p[0];
+#pragma unroll
+    for (int z = 1; z < 8; ++z)
+      if (z < n_parts) {
+        acc.x += p[z].x; acc.y += p[z].y; acc.z += p[z].z; acc.w += p[z].w;
+      }
+    for (int z = 8; z < n_parts; ++z) {
+      const float4 q = __ldcg(reinterpret_cast<const float4*>(part + z * part_stride + (size_t)m * d.W + col));
+      acc.x += q.x; acc.y += q.y; acc.z += q.z; acc.w += q.w;
+    }
     hv.x = fmaf(g.x, acc.x, hv.x);
     hv.y = fmaf(g.y, acc.y, hv.y);
     hv.z = fmaf(g.z, acc.z, hv.z);
     hv.w = fmaf(g.w, acc.w, hv.w);
     *reinterpret_cast<float4*>(hrow + col) = hv;
+    const float ss = block_sum(hv.x * hv.x + hv.y * hv.y + hv.z * hv.z + hv.w * hv.w, red);
+    const float rn = rsqrtf(ss / (float)d.W + d.eps);
+    store4<Act>(y + (size_t)m * d.W + col, hv.x * rn * (1.f + sc.x) + sh.x,
+                hv.y * rn * (1.f + sc.y) + sh.y, hv.z * rn * (1.f + sc.z) + sh.z,
+                hv.w * rn * (1.f + sc.w) + sh.w);
+    return;
+  }
+  float ss = 0.f;
+  for (int cc = col; cc < d.W; cc += blockDim.x * 4) {
+    float4 acc = __ldcg(reinterpret_cast<const float4*>(part + (size_t)m * d.W + cc));
+    for (int z = 1; z < n_parts; ++z) {
+      const float4 q =
+          __ldcg(reinterpret_cast<const float4*>(part + z * part_stride + (size_t)m * d.W + cc));
+      acc.x += q.x; acc.y += q.y; acc.z += q.z; acc.w += q.w;
+    }
+    const float4 g = *reinterpret_cast<const float4*>(mrow + gate_off + cc);
+    float4 hv = *reinterpret_cast<const float4*>(hrow + cc);
+    hv.x = fmaf(g.x, acc.x, hv.x);
+    hv.y = fmaf(g.y, acc.y, hv.y);
+    hv.z = fmaf(g.z, acc.z, hv.z);
+    hv.w = fmaf(g.w, acc.w, hv.w);
+    *reinterpret_cast<float4*>(hrow + cc) = hv;
     ss += hv.x * hv.x + hv.y * hv.y + hv.z * hv.z + hv.w * hv.w;
   }
   ss = block_sum(ss, red);

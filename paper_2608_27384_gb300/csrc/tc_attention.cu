@@ -249,28 +249,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld32_nowait(tO + lane_off + c0, o0);
       tmem_ld32_nowait(tO + lane_off + c0 + 32, o1);
       tmem_ld_wait();
-      if (valid) {
-        if (nsplit == 1) {
-          const float inv = l > 0.f ? 1.f / l : 0.f;
-          bf16* dst = (bf16*)a.out + (size_t)grow * kDH + c0;
+      // P, Q and the K/V ring are dead once O is complete: each warp stages its
+      // 32 rows there for coalesced stores
+      uint8_t* stage = smem + (warp - 2) * (32 * 272);
+      if (nsplit == 1) {
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        uint4 pk[8];
 #pragma unroll
-          for (int i = 0; i < 64; i += 8) {
-            float v[8];
+        for (int i = 0; i < 8; ++i) {
+          float v[8];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) v[u] = __uint_as_float(ov[i + u]) * inv;
-            *reinterpret_cast<uint4*>(dst + i) = pack_bf16x8(v);
-          }
-        } else {
-          float* po = a.part_o + (((size_t)gtile * a.max_splits + split) * kRows + row) * kDH + c0;
-#pragma unroll
-          for (int i = 0; i < 64; i += 4)
-            __stcg(reinterpret_cast<float4*>(po + i),
-                   make_float4(__uint_as_float(ov[i]), __uint_as_float(ov[i + 1]),
-                               __uint_as_float(ov[i + 2]), __uint_as_float(ov[i + 3])));
-          if (g == 0)
-            __stcg(a.part_ml + ((size_t)gtile * a.max_splits + split) * kRows + row,
-                   make_float2(mx, l));
+          for (int u = 0; u < 8; ++u) v[u] = __uint_as_float(ov[8 * i + u]) * inv;
+          pk[i] = pack_bf16x8(v);
         }
+        warp_store_rows<128>(stage, pk, valid ? (bf16*)a.out + (size_t)grow * kDH + c0 : nullptr,
+                             lane);
+      } else {
+        uint4 pk[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) pk[i] = make_uint4(ov[4 * i], ov[4 * i + 1], ov[4 * i + 2], ov[4 * i + 3]);
+        float* po = a.part_o + (((size_t)gtile * a.max_splits + split) * kRows + row) * kDH + c0;
+        warp_store_rows<256>(stage, pk, valid ? po : nullptr, lane);
+        if (valid && g == 0)
+          __stcg(a.part_ml + ((size_t)gtile * a.max_splits + split) * kRows + row,
+                 make_float2(mx, l));
       }
     }
   }

@@ -36,20 +36,25 @@ struct GemmCfg {
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
 };
 
-__device__ __forceinline__ void store_f32x32(float* dst, const float (&v)[32]) {
+__device__ __forceinline__ void pack_f32x32(const float (&v)[32], uint4 (&u)[8]) {
 #pragma unroll
-  for (int i = 0; i < 32; i += 4)
-    *reinterpret_cast<float4*>(dst + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+  for (int i = 0; i < 8; ++i)
+    u[i] = make_uint4(__float_as_uint(v[4 * i]), __float_as_uint(v[4 * i + 1]),
+                      __float_as_uint(v[4 * i + 2]), __float_as_uint(v[4 * i + 3]));
 }
 
-__device__ __forceinline__ void store_bf16x32(bf16* dst, const float (&v)[32]) {
+__device__ __forceinline__ void pack_bf16x32(const float (&v)[32], uint4 (&u)[4]) {
 #pragma unroll
-  for (int i = 0; i < 32; i += 8) *reinterpret_cast<uint4*>(dst + i) = pack_bf16x8(&v[i]);
+  for (int i = 0; i < 4; ++i) u[i] = pack_bf16x8(&v[8 * i]);
 }
 
+// Epilogue of one output row per thread; `stage` is this warp's private shared
+// memory (32 * 144 bytes): every 32-column chunk is stored through it with
+// coalesced 16-byte stores (warp_store_rows) while the next chunk is read from
+// TMEM.
 template <int BN, int MODE>
 __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, int m, int M,
-                                              int n0, int split) {
+                                              int n0, int split, uint8_t* stage, int lane) {
   const bool ok = m < M;
   if constexpr (MODE == GEMM_BIAS_F32 || MODE == GEMM_BIAS_SILU_BF16 ||
                 MODE == GEMM_PARTIAL_F32) {
@@ -57,20 +62,29 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
     for (int c = 0; c < BN; c += 32) {
       float v[32];
       tmem_ld32(trow + c, v);
-      if (!ok) continue;
       if constexpr (MODE == GEMM_PARTIAL_F32) {
-        float* dst = (float*)ep.out + split * ep.split_stride + (size_t)m * ep.ldo + n0 + c;
-        store_f32x32(dst, v);
+        uint4 u[8];
+        pack_f32x32(v, u);
+        float* dst = ok ? (float*)ep.out + split * ep.split_stride + (size_t)m * ep.ldo + n0 + c
+                        : nullptr;
+        warp_store_rows<128>(stage, u, dst, lane);
       } else {
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
           v[i] += __ldg(ep.bias + n0 + c + i);
           if constexpr (MODE == GEMM_BIAS_SILU_BF16) v[i] = silu_f(v[i]);
         }
-        if constexpr (MODE == GEMM_BIAS_F32)
-          store_f32x32((float*)ep.out + (size_t)m * ep.ldo + n0 + c, v);
-        else
-          store_bf16x32((bf16*)ep.out + (size_t)m * ep.ldo + n0 + c, v);
+        if constexpr (MODE == GEMM_BIAS_F32) {
+          uint4 u[8];
+          pack_f32x32(v, u);
+          warp_store_rows<128>(stage, u, ok ? (float*)ep.out + (size_t)m * ep.ldo + n0 + c : nullptr,
+                               lane);
+        } else {
+          uint4 u[4];
+          pack_bf16x32(v, u);
+          warp_store_rows<64>(stage, u, ok ? (bf16*)ep.out + (size_t)m * ep.ldo + n0 + c : nullptr,
+                              lane);
+        }
       }
     }
   } else if constexpr (MODE == GEMM_GEGLU) {
@@ -81,10 +95,12 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
       float g[32], u[32];
       tmem_ld32(trow + c, g);
       tmem_ld32(trow + half + c, u);
-      if (!ok) continue;
 #pragma unroll
       for (int i = 0; i < 32; ++i) g[i] = gelu_tanh_f(g[i]) * u[i];
-      store_bf16x32((bf16*)ep.out + (size_t)m * ep.ldo + n0 / 2 + c, g);
+      uint4 pk[4];
+      pack_bf16x32(g, pk);
+      warp_store_rows<64>(stage, pk, ok ? (bf16*)ep.out + (size_t)m * ep.ldo + n0 / 2 + c : nullptr,
+                          lane);
     }
   } else if constexpr (MODE == GEMM_QKV_ROPE) {
     // Weight rows are permuted so that tile column c < BN/2 holds head dim
@@ -116,9 +132,8 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
       float x1[32], x2[32];
       tmem_ld32(trow + c, x1);
       tmem_ld32(trow + half + c, x2);
-      if (!ok) continue;
       const int d0 = tj * half + c;
-      if (rotate) {
+      if (ok && rotate) {
 #pragma unroll
         for (int i = 0; i < 32; i += 2) {
           const float a0 = x1[i], b0 = x2[i], a1 = x1[i + 1], b1 = x2[i + 1];
@@ -128,8 +143,11 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
           x2[i + 1] = b1 * cs[i / 2].z + a1 * cs[i / 2].w;
         }
       }
-      store_bf16x32(dst + d0, x1);
-      store_bf16x32(dst + d0 + dh / 2, x2);
+      uint4 p1[4], p2[4];
+      pack_bf16x32(x1, p1);
+      pack_bf16x32(x2, p2);
+      warp_store_rows<64>(stage, p1, ok ? dst + d0 : nullptr, lane);
+      warp_store_rows<64>(stage, p2, ok ? dst + d0 + dh / 2 : nullptr, lane);
     }
   }
 }
@@ -223,8 +241,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool good = __all_sync(0xffffffffu, mbar_wait(acc_full, 0, ep.err, KERR_WAIT_MMA));
     tc_fence_after();
     if (good && nkb > 0) {
+      // all MMAs (and so all TMA loads into the ring) are complete: the ring's
+      // first stage is free to stage this warp's coalesced stores
       const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
-      gemm_epilogue<BN, MODE>(ep, trow, m0 + row, M, n0, split);
+      uint8_t* stage = smem + (warp - 2) * (32 * 144);
+      gemm_epilogue<BN, MODE>(ep, trow, m0 + row, M, n0, split, stage, lane);
     }
   }
   tc_fence_before();
