@@ -340,6 +340,21 @@ def main():
                  "share_of_profiled_step": t_us / prof_total, "peak_source": f"{peak_src} burst"})
     shares = {k: round(v[0] / prof_total, 4) for k, v in sorted(per_kind.items(),
                                                                 key=lambda kv: -kv[1][0])}
+    # every kernel kind against its own binding peak (same event-timed launches)
+    kernel_rooflines = {}
+    for k, (t_k, n_k) in per_kind.items():
+        if k not in costs:
+            continue
+        fl_k, by_k = costs[k]
+        avg_k = t_k / n_k * 1e-6
+        tensor = fl_k / tc >= by_k / bw
+        ach = (fl_k / avg_k / 1e12) if tensor else (by_k / avg_k / 1e9)
+        kernel_rooflines[k] = {"bound": "tensor" if tensor else "hbm",
+                               "avg_launch_us": round(t_k / n_k, 3),
+                               "achieved": round(ach, 2),
+                               "unit": "TFLOP/s" if tensor else "GB/s",
+                               "frac": round(ach / (peaks["bf16_tflops"] if tensor
+                                                    else peaks["hbm_gbs"]), 4)}
 
     flops, nbytes = step_costs(wl, B)
     t_roof = max(flops / tc, nbytes / bw)
@@ -368,6 +383,11 @@ def main():
                         "d2h_bytes_per_step": d2h, "steps": e2e_steps},
                 "gpu_launches": launches_per_step * args.steps,
                 "roofline": roof, "step_roofline": step_roof, "kernel_shares": shares,
+                "kernel_rooflines": kernel_rooflines,
+                "profile_note": "per-kernel times: CUDA events between the kernels of a "
+                                "captured profiling graph (event nodes serialise the "
+                                "kernels, so they include launch gaps the timed step "
+                                "hides)",
                 "cpu_baseline": cpu}
         print(json.dumps(line))
     if dist is not None:

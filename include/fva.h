@@ -283,12 +283,13 @@ typedef struct fva_kernel_time {
 
 /*
  * One step exactly like fva_step (same kernels, same results, advances the step
- * index) but launched kernel by kernel with a CUDA event recorded before every
- * launch and after the last; waits for the stream, then writes one record per
- * launch, in launch order, to records[0 .. *n_records).  Each duration spans
- * from the launch's own event to the next event on the stream, i.e. the kernel
- * plus the launch gap after it.  Errors: as fva_step, plus INVALID_ARG when
- * max_records is smaller than the number of launches.
+ * index), replayed from a separately captured CUDA graph that has an event node
+ * before every kernel and after the last (the events serialise the kernels, so
+ * the overlap programmatic dependent launch gives the normal step is lost).
+ * Waits for the stream, then writes one record per launch, in launch order, to
+ * records[0 .. *n_records); each duration spans from the launch's event to the
+ * next one.  Errors: as fva_step, plus INVALID_ARG when max_records is smaller
+ * than the number of launches.
  */
 fva_status fva_step_profile(fva_handle* h, float* buffer, const float* noise_levels,
                             float* out_chunk, int32_t batch, fva_kernel_time* records,

@@ -166,6 +166,12 @@ struct fva_handle {
   cudaEvent_t err_ev = nullptr;
   bool err_pending = false;
   uint64_t polls = 0;
+  // profiling graph (fva_step_profile): events between kernels
+  std::vector<cudaEvent_t> prof_events;
+  cudaGraphExec_t prof_exec = nullptr;
+  int prof_batch = 0;
+  float *prof_buf = nullptr, *prof_out = nullptr;
+  std::vector<int> prof_kind, prof_layer;
   // graphs
   cudaStream_t cap_stream = nullptr;
   std::vector<GraphEntry> graphs;
@@ -207,6 +213,10 @@ void release(fva_handle* h) {
   cudaDeviceSynchronize();
   for (auto& g : h->graphs) cudaGraphExecDestroy(g.exec);
   h->graphs.clear();
+  if (h->prof_exec) cudaGraphExecDestroy(h->prof_exec);
+  h->prof_exec = nullptr;
+  for (auto e : h->prof_events) cudaEventDestroy(e);
+  h->prof_events.clear();
   for (void* p : h->allocs) cudaFree(p);
   h->allocs.clear();
   if (h->warena) cudaFree(h->warena);
@@ -390,7 +400,7 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
     d.K = h->K;
     d.A = h->A;
     d.W = h->W;
-    if (sizeof(float) * ((size_t)2 * d.K * d.A + (size_t)(d.K + d.A) * 4) > 200 * 1024)
+    if (sizeof(float) * ((size_t)18 * d.K * d.A + (size_t)(d.K + d.A) * 4) > 200 * 1024)
       return fail(FVA_ERR_UNSUPPORTED, "n_chunks * action_dim too large for the final kernel");
     CUDA_TRY(final_init(d));
   }
@@ -623,6 +633,8 @@ extern "C" fva_status fva_load_weights(fva_handle* h, const void* const* tensors
   // upload into a fresh arena (replacing any previous weights)
   for (auto& g : h->graphs) cudaGraphExecDestroy(g.exec);
   h->graphs.clear();
+  if (h->prof_exec) cudaGraphExecDestroy(h->prof_exec);
+  h->prof_exec = nullptr;
   if (h->warena) cudaFree(h->warena);
   h->warena = nullptr;
   h->weights_loaded = false;
@@ -720,25 +732,33 @@ struct StepTrace {
   float* out = nullptr;
 };
 
-// Event before every launch (kernel profiling mode of fva_step_profile).
+// Event before every launch (kernel profiling mode of fva_step_profile).  The
+// events come from a pool owned by the handle and are recorded while the
+// profiling graph is captured, so every replay re-records them between kernels.
 struct StepProfile {
-  std::vector<cudaEvent_t> events;
+  std::vector<cudaEvent_t>* pool = nullptr;
+  size_t used = 0;
   std::vector<int> kind, layer;
   cudaError_t err = cudaSuccess;
   void mark(int k, int l, cudaStream_t s) {
-    cudaEvent_t e;
-    cudaError_t r = cudaEventCreate(&e);
-    if (r == cudaSuccess) r = cudaEventRecord(e, s);
+    if (used == pool->size()) {
+      cudaEvent_t e;
+      cudaError_t r = cudaEventCreate(&e);
+      if (r != cudaSuccess) {
+        err = r;
+        return;
+      }
+      pool->push_back(e);
+    }
+    // an external record is captured as an event-record node that every replay re-records
+    cudaError_t r = cudaEventRecordWithFlags((*pool)[used], s, cudaEventRecordExternal);
     if (r != cudaSuccess) {
       err = r;
       return;
     }
-    events.push_back(e);
+    ++used;
     kind.push_back(k);
     layer.push_back(l);
-  }
-  ~StepProfile() {
-    for (auto e : events) cudaEventDestroy(e);
   }
 };
 
@@ -1082,13 +1102,42 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
   if (fresh)
     CUDA_TRY(cudaMemcpyAsync(h->fresh, opts->fresh_noise,
                              sizeof(float) * batch * h->H * h->A, cudaMemcpyDeviceToDevice, s));
-  if (prof || (opts && opts->trace_layer >= 0) || (h->cfg.flags & FVA_FLAG_NO_GRAPH)) {
+  if (prof) {
+    if (!h->prof_exec || h->prof_batch != batch || h->prof_buf != buffer ||
+        h->prof_out != out_chunk) {
+      if (h->prof_exec) cudaGraphExecDestroy(h->prof_exec);
+      h->prof_exec = nullptr;
+      prof->pool = &h->prof_events;
+      cudaGraph_t graph;
+      CUDA_TRY(cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal));
+      st = enqueue_step(h, batch, buffer, out_chunk, fresh, StepTrace{}, h->cap_stream, prof);
+      cudaError_t e = cudaStreamEndCapture(h->cap_stream, &graph);
+      if (st != FVA_OK) {
+        if (e == cudaSuccess) cudaGraphDestroy(graph);
+        return st;
+      }
+      CUDA_TRY(e);
+      e = cudaGraphInstantiate(&h->prof_exec, graph, 0);
+      cudaGraphDestroy(graph);
+      CUDA_TRY(e);
+      h->prof_batch = batch;
+      h->prof_buf = buffer;
+      h->prof_out = out_chunk;
+      h->prof_kind = prof->kind;
+      h->prof_layer = prof->layer;
+    }
+    prof->pool = &h->prof_events;
+    prof->used = h->prof_kind.size();
+    prof->kind = h->prof_kind;
+    prof->layer = h->prof_layer;
+    CUDA_TRY(cudaGraphLaunch(h->prof_exec, s));
+  } else if ((opts && opts->trace_layer >= 0) || (h->cfg.flags & FVA_FLAG_NO_GRAPH)) {
     StepTrace tr;
     if (opts && opts->trace_layer >= 0) {
       tr.layer = opts->trace_layer;
       tr.out = opts->trace_out;
     }
-    if ((st = enqueue_step(h, batch, buffer, out_chunk, fresh, tr, s, prof)) != FVA_OK) return st;
+    if ((st = enqueue_step(h, batch, buffer, out_chunk, fresh, tr, s)) != FVA_OK) return st;
   } else {
     cudaGraphExec_t exec;
     if ((st = get_graph(h, batch, buffer, out_chunk, fresh, &exec)) != FVA_OK) return st;
@@ -1132,11 +1181,11 @@ extern "C" fva_status fva_step_profile(fva_handle* h, float* buffer, const float
   if (st != FVA_OK) return st;
   DeviceGuard guard(h->device);
   CUDA_TRY(cudaStreamSynchronize((cudaStream_t)stream));
-  const int n = (int)prof.events.size() - 1;
+  const int n = (int)prof.used - 1;
   if (n > max_records) return fail(FVA_ERR_INVALID_ARG, "max_records %d < %d", max_records, n);
   for (int i = 0; i < n; ++i) {
     float ms = 0.f;
-    CUDA_TRY(cudaEventElapsedTime(&ms, prof.events[i], prof.events[i + 1]));
+    CUDA_TRY(cudaEventElapsedTime(&ms, h->prof_events[i], h->prof_events[i + 1]));
     records[i].kind = prof.kind[i];
     records[i].layer = prof.layer[i];
     records[i].microseconds = ms * 1000.f;

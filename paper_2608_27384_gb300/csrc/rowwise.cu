@@ -312,6 +312,7 @@ __global__ void __launch_bounds__(kVelThreads)
   float* ws = ys + d.K * wchunk;     // [wchunk][A]
   float* xs = ws + wchunk * d.A;     // [K][A] buffer values of this column
   float* vs = xs + KA;               // [K][A] velocities
+  float* red = vs + KA;              // [16][K][A] partial sums of the w-range groups
   if (threadIdx.x == 0) {
     mbar_init(&bar, 1);
     fence_barrier_init();
@@ -339,17 +340,52 @@ __global__ void __launch_bounds__(kVelThreads)
     }
     mbar_wait(&bar, phase, nullptr, 0);
     phase ^= 1u;
-    for (int i = threadIdx.x; i < KA; i += blockDim.x) {
-      const int k = i / d.A, a = i % d.A;
-      const float* yk = ys + k * wchunk;
-      float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
-      for (int w = 0; w < wchunk; w += 4) {
-        acc0 = fmaf(yk[w], ws[w * d.A + a], acc0);
-        acc1 = fmaf(yk[w + 1], ws[(w + 1) * d.A + a], acc1);
-        acc2 = fmaf(yk[w + 2], ws[(w + 2) * d.A + a], acc2);
-        acc3 = fmaf(yk[w + 3], ws[(w + 3) * d.A + a], acc3);
+    if (d.A % 4 == 0) {
+      // thread = (w-range group, k, 4 consecutive a): 16-byte shared loads, each
+      // y_F value reused for 4 outputs; groups split the w range and their
+      // partial sums are added in group order below
+      const int per = d.K * (d.A / 4);
+      const int groups = min((int)blockDim.x / per, 16);
+      const int span = ((wchunk / 4 + groups - 1) / groups) * 4;
+      const int t = threadIdx.x;
+      if (t < groups * per) {
+        const int gi = t / per, rem = t % per, k = rem / (d.A / 4), a4 = (rem % (d.A / 4)) * 4;
+        const int w0c = gi * span, w1c = min(wchunk, w0c + span);
+        const float* yk = ys + k * wchunk;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int w = w0c; w < w1c; w += 4) {
+          const float4 y4 = *reinterpret_cast<const float4*>(yk + w);
+          const float yv[4] = {y4.x, y4.y, y4.z, y4.w};
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const float4 wv = *reinterpret_cast<const float4*>(ws + (w + u) * d.A + a4);
+            acc.x = fmaf(yv[u], wv.x, acc.x);
+            acc.y = fmaf(yv[u], wv.y, acc.y);
+            acc.z = fmaf(yv[u], wv.z, acc.z);
+            acc.w = fmaf(yv[u], wv.w, acc.w);
+          }
+        }
+        *reinterpret_cast<float4*>(red + (size_t)gi * KA + k * d.A + a4) = acc;
       }
-      vs[i] += (acc0 + acc1) + (acc2 + acc3);
+      __syncthreads();
+      for (int i = threadIdx.x; i < KA; i += blockDim.x) {
+        float v = 0.f;
+        for (int gi = 0; gi < groups; ++gi) v += red[(size_t)gi * KA + i];
+        vs[i] += v;
+      }
+    } else {
+      for (int i = threadIdx.x; i < KA; i += blockDim.x) {
+        const int k = i / d.A, a = i % d.A;
+        const float* yk = ys + k * wchunk;
+        float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
+        for (int w = 0; w < wchunk; w += 4) {
+          acc0 = fmaf(yk[w], ws[w * d.A + a], acc0);
+          acc1 = fmaf(yk[w + 1], ws[(w + 1) * d.A + a], acc1);
+          acc2 = fmaf(yk[w + 2], ws[(w + 2) * d.A + a], acc2);
+          acc3 = fmaf(yk[w + 3], ws[(w + 3) * d.A + a], acc3);
+        }
+        vs[i] += (acc0 + acc1) + (acc2 + acc3);
+      }
     }
   }
   __syncthreads();
@@ -376,14 +412,14 @@ __global__ void __launch_bounds__(kVelThreads)
 // Largest W-chunk (a divisor of W, multiple of 4) whose staging fits ~200 KB.
 // Every bulk copy then starts 16-byte aligned (W and the chunk are multiples of 4).
 static int vel_chunk(const StepDims& d) {
-  const size_t budget = 200 * 1024 - sizeof(float) * 2 * d.K * d.A;
+  const size_t budget = 200 * 1024 - sizeof(float) * 18 * d.K * d.A;
   int c = d.W;
   while (c > 4 && (sizeof(float) * (size_t)(d.K + d.A) * c > budget || d.W % c || c % 4)) --c;
   return c;
 }
 
 static size_t vel_smem_bytes(const StepDims& d) {
-  return sizeof(float) * ((size_t)2 * d.K * d.A + (size_t)(d.K + d.A) * vel_chunk(d));
+  return sizeof(float) * ((size_t)18 * d.K * d.A + (size_t)(d.K + d.A) * vel_chunk(d));
 }
 
 cudaError_t final_init(const StepDims& d) {

@@ -285,3 +285,32 @@ def test_step_before_weights_and_prefix():
         assert e.value.name == "FVA_ERR_STATE" and "prefix" in str(e.value)
     finally:
         fva.fva_destroy(h)
+
+
+def test_step_profile_matches_step_and_counts_launches():
+    import torch
+    import paper_2608_27384_gb300 as fva
+    wl = WL.small_bf16_workload(n_chunks=4, prefix_lens=[600])
+    case = Case(wl)
+    try:
+        d_a, d_b = case.dev(case.buf), case.dev(case.buf)
+        o_a = torch.empty((1, wl.chunk_tokens, wl.action_dim), device="cuda")
+        o_b = torch.empty_like(o_a)
+        fva.fva_set_step_index(case.handle, 5)
+        fva.fva_step(case.handle, d_a, case.tau, o_a, 1)
+        fva.fva_set_step_index(case.handle, 5)
+        recs = fva.fva_step_profile(case.handle, d_b, case.tau, o_b, 1)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(o_a.cpu().numpy(), o_b.cpu().numpy())
+        np.testing.assert_array_equal(d_a.cpu().numpy(), d_b.cpu().numpy())
+        kinds = [k for k, _, _ in recs]
+        L = wl.n_layers
+        # time embedding, 2 time-MLP layers, FiLM, embed+norm; per layer QKV,
+        # attention, split merge (prefix 600 + 200 keys > 256), O, norm, gate/up,
+        # down, norm (last layer: final norm); velocity
+        assert len(recs) == 5 + 8 * L + 1, kinds
+        assert kinds.count("attention") == L and kinds.count("attn_merge") == L
+        assert kinds[-1] == "velocity" and kinds[-2] == "final_norm"
+        assert all(us > 0 for _, _, us in recs)
+    finally:
+        case.close()
