@@ -238,8 +238,8 @@ fva_status fva_chunk_attention(fva_handle* h, const void* q, const void* k, cons
  *
  * Same inputs, output and numerics as fva_chunk_attention, with the shapes passed
  * explicitly (head_dim must be 256, n_q_heads one of 1, 2, 4, 8, 16).  The split-KV
- * scratch is a fixed array inside the library: 256 slots of 128 x 256 fp32 plus
- * row statistics (32 MiB + 256 KiB), kept by every GPU that loads the library
+ * scratch is a fixed array inside the library: 256 slots of 128 x 256 bf16 plus
+ * row statistics (16 MiB + 256 KiB), kept by every GPU that loads the library
  * until the process exits.  A call needs
  *   batch * ceil(K*H*n_q_heads / 128) * ceil(kv_rows / 256)
  * slots (and ceil(kv_rows / 256) <= 32); larger calls return FVA_ERR_INVALID_ARG.

@@ -30,13 +30,13 @@ constexpr int kRowsPerSlot = 128;
 constexpr int kDH = 256;
 constexpr int kMaxDevices = 64;
 
-static __device__ __align__(256) float g_part_o[(size_t)kNoAllocSlots * kRowsPerSlot * kDH];
+static __device__ __align__(256) bf16 g_part_o[(size_t)kNoAllocSlots * kRowsPerSlot * kDH];
 static __device__ __align__(256) float2 g_part_ml[(size_t)kNoAllocSlots * kRowsPerSlot];
 
 struct DeviceScratch {
   std::once_flag once;
   cudaError_t status = cudaErrorNotReady;
-  float* part_o = nullptr;
+  bf16* part_o = nullptr;
   float2* part_ml = nullptr;
 };
 DeviceScratch g_dev[kMaxDevices];

@@ -149,7 +149,7 @@ struct fva_handle {
   float *mod = nullptr, *h = nullptr, *part = nullptr, *c32 = nullptr, *vel = nullptr;
   float* yF = nullptr;  // [Mmax, W] fp32 output of the final FiLM RMSNorm
   float* fresh = nullptr;
-  float* att_part_o = nullptr;
+  __nv_bfloat16* att_part_o = nullptr;
   float2* att_part_ml = nullptr;
   int* err_dev = nullptr;
   CUtensorMap m_temb, m_t1, m_cond, m_y, m_attn, m_mlp, m_q, m_k, m_v;

@@ -132,7 +132,7 @@ cudaError_t launch_tc_gemm(int bn, int mode, const CUtensorMap* a, const CUtenso
 struct AttnArgs {
   const int* prefix_len;
   void* out;            // bf16 [Bmax*T*nq, 256]
-  float* part_o;        // [B*tiles, max_splits, 128, 256]
+  void* part_o;         // bf16 [B*tiles, max_splits, 128, 256]: per-split O / l
   float2* part_ml;      // [B*tiles, max_splits, 128]
   int T, H, nq, S_cap, tiles_per_req, max_splits;
   int kv_row0;          // first KV row of this layer in the 2D view

@@ -16,12 +16,16 @@
 //               S = Q K^T per key block (M=128, N=64, K=16 steps over dh), and,
 //               after the softmax, O = P V (M=128, N=256, MN-major V);
 //   warps 2..17 softmax + epilogue, four threads per query row (one per
-//               64-key block / 64 head-dim columns): exact row max over the
-//               split's visible keys, P = exp(S - max) written as bf16 over the Q
-//               tile (Q is dead once S is complete), row sum; then O from TMEM.
-// A tile with one split writes O / l as bf16.  Otherwise each split writes its
-// unnormalised (O, max, sum) to scratch and attn_merge_kernel combines the
-// splits of every row in split order (deterministic) and writes bf16.
+//               64-key block / 64 head-dim columns).  As soon as its block of S
+//               is in TMEM a thread takes the block's row max over visible keys
+//               and writes P = exp(S - block max) as bf16 over the Q tile (Q is
+//               dead once S is complete); after the four threads of a row
+//               exchange maxima it rescales its P block by exp(block max - row
+//               max) in place, so the exponentials overlap the S MMAs of later
+//               blocks.  Then O is read from TMEM.
+// A tile with one split writes O / l as bf16.  Otherwise each split writes O / l
+// (bf16) and its (max, sum) to scratch and attn_merge_kernel combines the splits
+// of every row in split order (deterministic) and writes bf16.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -73,10 +77,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* q_full = bars + 0;
   uint64_t* kv_full = bars + 1;   // [4]
   uint64_t* kv_empty = bars + 5;  // [4]
-  uint64_t* s_full = bars + 9;
-  uint64_t* p_full = bars + 10;
-  uint64_t* o_full = bars + 11;
-  uint32_t* tmem_slot = (uint32_t*)(bars + 12);
+  uint64_t* s_full = bars + 9;    // [4]: block g of S is in TMEM
+  uint64_t* p_full = bars + 13;
+  uint64_t* o_full = bars + 14;
+  uint32_t* tmem_slot = (uint32_t*)(bars + 15);
   float* xmax = (float*)(bars + 128);   // [4][128] per-block row max
   float* xsum = xmax + 4 * kRows;       // [4][128] per-block row sum
 
@@ -87,7 +91,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&kv_full[s], 1);
       mbar_init(&kv_empty[s], 1);
     }
-    mbar_init(s_full, 1);
+    for (int g = 0; g < kBlocksPerSplit; ++g) mbar_init(&s_full[g], 1);
     mbar_init(p_full, kSoftmaxThreads);
     mbar_init(o_full, 1);
     fence_barrier_init();
@@ -158,8 +162,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         umma_bf16(tS + it * kKB, ad, bd, idesc_s, ks > 0 ? 1u : 0u);
       }
       umma_commit(&kv_empty[s]);
+      umma_commit(&s_full[it]);
     }
-    if (good) umma_commit(s_full);
     if (good) good = mbar_wait(p_full, 0, a.err, KERR_WAIT_SYNC);
     tc_fence_after();
     for (int j = 0; good && j < nblk; ++j) {
@@ -191,34 +195,27 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
     const bool has_blk = g < nblk;
     const int key0 = (kb0 + g) * kKB;
-    bool good = __all_sync(0xffffffffu, mbar_wait(s_full, 0, a.err, KERR_WAIT_MMA));
+    // this thread's block of S (threads of absent blocks wait for the last block,
+    // which every thread needs before P may overwrite Q)
+    bool good = __all_sync(0xffffffffu, mbar_wait(&s_full[has_blk ? g : nblk - 1], 0, a.err,
+                                                  KERR_WAIT_MMA));
     tc_fence_after();
     float mx = -INFINITY, l = 0.f;
-    uint32_t sv[64];
+    const int nvis = min(kKB, max(0, limit - key0));
+    uint4 pk[8];  // P of this block against the block's own max, bf16, logical order
     if (good && has_blk) {
+      uint32_t sv[64];
       uint32_t (&s0)[32] = *reinterpret_cast<uint32_t(*)[32]>(&sv[0]);
       uint32_t (&s1)[32] = *reinterpret_cast<uint32_t(*)[32]>(&sv[32]);
       tmem_ld32_nowait(tS + lane_off + g * kKB, s0);
       tmem_ld32_nowait(tS + lane_off + g * kKB + 32, s1);
       tmem_ld_wait();
-      if (key0 + kKB <= limit) {  // whole block visible
 #pragma unroll
-        for (int i = 0; i < 64; ++i) mx = fmaxf(mx, __uint_as_float(sv[i]));
-      } else {
+      for (int i = 0; i < 64; ++i)
+        if (i < nvis) mx = fmaxf(mx, __uint_as_float(sv[i]));
+      const float mscaled = mx > -INFINITY ? mx * a.scale_log2 : 0.f;
 #pragma unroll
-        for (int i = 0; i < 64; ++i)
-          if (key0 + i < limit) mx = fmaxf(mx, __uint_as_float(sv[i]));
-      }
-    }
-    xmax[g * kRows + row] = mx;
-    softmax_bar();
-    mx = fmaxf(fmaxf(xmax[row], xmax[kRows + row]), fmaxf(xmax[2 * kRows + row], xmax[3 * kRows + row]));
-    if (good && has_blk) {
-      const float mscaled = mx * a.scale_log2;
-      uint8_t* prow = sQP + g * (kRows * 128) + row * 128;
-      const int nvis = min(kKB, max(0, limit - key0));
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {  // 16-byte chunk c = keys 8c .. 8c+7
+      for (int c = 0; c < 8; ++c) {  // keys 8c .. 8c+7
         float p[8];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
@@ -228,17 +225,47 @@ __global__ void __launch_bounds__(kThreads, 1)
           l += pr;
           p[i] = pr;
         }
-        const int phys = c ^ (row & 7);  // 128-byte swizzle
-        *reinterpret_cast<uint4*>(prow + phys * 16) = pack_bf16x8(p);
+        pk[c] = pack_bf16x8(p);
       }
     }
+    xmax[g * kRows + row] = mx;
     xsum[g * kRows + row] = l;
+    // block maxima and sums of every row.  The threads of the last block (and of
+    // absent blocks) waited for the last S commit, which covers every S MMA, so
+    // past this barrier Q is dead for all threads and P may go over it.
+    softmax_bar();
+    float bm[kBlocksPerSplit];
+#pragma unroll
+    for (int j = 0; j < kBlocksPerSplit; ++j) bm[j] = xmax[j * kRows + row];
+    const float mrow = fmaxf(fmaxf(bm[0], bm[1]), fmaxf(bm[2], bm[3]));
+    // row sum over blocks, each block's sum scaled to the row max
+    l = 0.f;
+#pragma unroll
+    for (int j = 0; j < kBlocksPerSplit; ++j)
+      if (bm[j] > -INFINITY) l += xsum[j * kRows + row] * exp2f((bm[j] - mrow) * a.scale_log2);
+    if (good && has_blk) {
+      // P, rescaled to the row max, goes over Q, 128-byte swizzled
+      uint8_t* prow = sQP + g * (kRows * 128) + row * 128;
+      const float alpha = mx > -INFINITY ? exp2f((mx - mrow) * a.scale_log2) : 0.f;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        uint4 u = pk[c];
+        if (alpha != 1.f) {
+          __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+          for (int q2 = 0; q2 < 4; ++q2) {
+            const float2 f = __bfloat1622float2(h2[q2]);
+            h2[q2] = __floats2bfloat162_rn(f.x * alpha, f.y * alpha);
+          }
+        }
+        *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) * 16)) = u;
+      }
+    }
+    mx = mrow;
     fence_proxy_async_smem();
     mbar_arrive(p_full);
     if (good) good = __all_sync(0xffffffffu, mbar_wait(o_full, 0, a.err, KERR_WAIT_MMA));
     tc_fence_after();
-    softmax_bar();  // xsum complete
-    l = (xsum[row] + xsum[kRows + row]) + (xsum[2 * kRows + row] + xsum[3 * kRows + row]);
     const int gtile = r * a.tiles_per_req + tile;
     const int grow = qrow0 + row;  // global q row = (r*T + t) * nq + head
     const int c0 = g * 64;         // O columns of this thread
@@ -251,29 +278,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld_wait();
       // P, Q and the K/V ring are dead once O is complete: each warp stages its
       // 32 rows there for coalesced stores
-      uint8_t* stage = smem + (warp - 2) * (32 * 272);
-      if (nsplit == 1) {
-        const float inv = l > 0.f ? 1.f / l : 0.f;
-        uint4 pk[8];
+      uint8_t* stage = smem + (warp - 2) * (32 * 144);
+      // one split: the output row; several: this split's partial (O / l, with
+      // max and sum) for attn_merge_kernel
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      uint4 pk[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          float v[8];
+      for (int i = 0; i < 8; ++i) {
+        float v[8];
 #pragma unroll
-          for (int u = 0; u < 8; ++u) v[u] = __uint_as_float(ov[8 * i + u]) * inv;
-          pk[i] = pack_bf16x8(v);
-        }
-        warp_store_rows<128>(stage, pk, valid ? (bf16*)a.out + (size_t)grow * kDH + c0 : nullptr,
-                             lane);
-      } else {
-        uint4 pk[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) pk[i] = make_uint4(ov[4 * i], ov[4 * i + 1], ov[4 * i + 2], ov[4 * i + 3]);
-        float* po = a.part_o + (((size_t)gtile * a.max_splits + split) * kRows + row) * kDH + c0;
-        warp_store_rows<256>(stage, pk, valid ? po : nullptr, lane);
-        if (valid && g == 0)
-          __stcg(a.part_ml + ((size_t)gtile * a.max_splits + split) * kRows + row,
-                 make_float2(mx, l));
+        for (int u = 0; u < 8; ++u) v[u] = __uint_as_float(ov[8 * i + u]) * inv;
+        pk[i] = pack_bf16x8(v);
       }
+      const size_t prow_idx = ((size_t)gtile * a.max_splits + split) * kRows + row;
+      bf16* dst = nsplit == 1 ? (bf16*)a.out + (size_t)grow * kDH + c0
+                              : (bf16*)a.part_o + prow_idx * kDH + c0;
+      warp_store_rows<128>(stage, pk, valid ? dst : nullptr, lane);
+      if (nsplit > 1 && valid && g == 0) __stcg(a.part_ml + prow_idx, make_float2(mx, l));
     }
   }
   tc_fence_before();
@@ -284,9 +305,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// Combine the key splits of every query row of tiles that have more than one:
-// o = sum_s 2^((m_s - m) c) O_s / sum_s 2^((m_s - m) c) l_s, m = max over splits
-// with keys, c = log2(e)/sqrt(dh); splits in order.  One warp per row, 8 dh
+// Combine the key splits of every query row of tiles that have more than one.
+// Split s stored o_s = O_s / l_s with its (m_s, l_s); with w_s = 2^((m_s - m) c) l_s,
+// m = max over splits with keys, c = log2(e)/sqrt(dh):  o = sum_s w_s o_s / sum_s w_s,
+// splits in order.  One warp per row, 8 dh
 // values per lane.
 __global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -307,28 +329,30 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
   float2 ml = make_float2(-INFINITY, 0.f);
   if (lane < nsplit) ml = __ldcg(a.part_ml + (tbase + lane) * kRows + row);
   float m_all = warp_max(ml.y > 0.f ? ml.x : -INFINITY);
-  const float w = ml.y > 0.f ? exp2f((ml.x - m_all) * a.scale_log2) : 0.f;
-  const float inv = 1.f / warp_sum(w * ml.y);
+  // each split stored O_s / l_s; its weight is 2^((m_s - m) c) l_s
+  const float w = ml.y > 0.f ? exp2f((ml.x - m_all) * a.scale_log2) * ml.y : 0.f;
+  const float inv = 1.f / warp_sum(w);
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   for (int s0 = 0; s0 < nsplit; s0 += 8) {  // up to 8 splits' loads in flight
-    float4 x[8][2];
+    uint4 x[8];
     float ws[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       ws[u] = __shfl_sync(0xffffffffu, w, (s0 + u) & 31);
-      if (s0 + u < nsplit) {
-        const float* po = a.part_o + ((tbase + s0 + u) * kRows + row) * kDH + lane * 8;
-        x[u][0] = __ldcg(reinterpret_cast<const float4*>(po));
-        x[u][1] = __ldcg(reinterpret_cast<const float4*>(po + 4));
-      }
+      if (s0 + u < nsplit)
+        x[u] = __ldcg(reinterpret_cast<const uint4*>(
+            (const bf16*)a.part_o + ((tbase + s0 + u) * kRows + row) * kDH + lane * 8));
     }
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       if (s0 + u < nsplit) {
-        acc[0] = fmaf(ws[u], x[u][0].x, acc[0]); acc[1] = fmaf(ws[u], x[u][0].y, acc[1]);
-        acc[2] = fmaf(ws[u], x[u][0].z, acc[2]); acc[3] = fmaf(ws[u], x[u][0].w, acc[3]);
-        acc[4] = fmaf(ws[u], x[u][1].x, acc[4]); acc[5] = fmaf(ws[u], x[u][1].y, acc[5]);
-        acc[6] = fmaf(ws[u], x[u][1].z, acc[6]); acc[7] = fmaf(ws[u], x[u][1].w, acc[7]);
+        const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&x[u]);
+#pragma unroll
+        for (int q2 = 0; q2 < 4; ++q2) {
+          const float2 f = __bfloat1622float2(h2[q2]);
+          acc[2 * q2] = fmaf(ws[u], f.x, acc[2 * q2]);
+          acc[2 * q2 + 1] = fmaf(ws[u], f.y, acc[2 * q2 + 1]);
+        }
       }
     }
   }
