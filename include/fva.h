@@ -101,6 +101,10 @@ typedef struct fva_handle fva_handle;
  * activations, scratch) and zero-fills them.  *out receives the handle.
  * Errors: INVALID_ARG (bad field), UNSUPPORTED (shape outside the dtype's
  * kernels), OOM, CUDA.  Nothing is allocated when an error is returned.
+ * Environment: FVA_BLOCK_KERNEL=1 (read here) makes bf16 steps run each layer's
+ * post-attention part as one persistent kernel (FVA_K_BLOCK) instead of one
+ * launch per operation, where the sizes allow it (width a multiple of 256 up to
+ * 1024); results agree within the bf16 tolerances, not bit for bit.
  */
 fva_status fva_create(const fva_config* cfg, fva_handle** out);
 
@@ -272,7 +276,10 @@ typedef enum fva_kernel_kind {
   FVA_K_FINAL = 10,          /* last gated residual + final FiLM RMSNorm (fp32 out)  */
   FVA_K_ATTN_MERGE = 11,     /* combination of the attention's key splits            */
   FVA_K_VELOCITY = 12,       /* out-projection + Euler + emit + roll + tail          */
-  FVA_K_COUNT = 13
+  FVA_K_BLOCK = 13,          /* fused post-attention part of a layer: O-projection,
+                                norm 2, gate/up, down, then the next layer's norm 1
+                                and QKV projection (or the final norm)               */
+  FVA_K_COUNT = 14
 } fva_kernel_kind;
 
 typedef struct fva_kernel_time {

@@ -1,0 +1,128 @@
+// Epilogues of the tcgen05 GEMMs: one output row per thread, read from TMEM in
+// 32-column chunks and stored through a per-warp shared-memory stage with
+// coalesced 16-byte stores.  Shared by the per-op GEMM kernel and the fused
+// block kernel.
+#pragma once
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace fva {
+
+__device__ __forceinline__ void pack_f32x32(const float (&v)[32], uint4 (&u)[8]) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    u[i] = make_uint4(__float_as_uint(v[4 * i]), __float_as_uint(v[4 * i + 1]),
+                      __float_as_uint(v[4 * i + 2]), __float_as_uint(v[4 * i + 3]));
+}
+
+__device__ __forceinline__ void pack_bf16x32(const float (&v)[32], uint4 (&u)[4]) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) u[i] = pack_bf16x8(&v[8 * i]);
+}
+
+// Epilogue of one output row per thread; `stage` is this warp's private shared
+// memory (32 * 144 bytes): every 32-column chunk is stored through it with
+// coalesced 16-byte stores (warp_store_rows) while the next chunk is read from
+// TMEM.
+template <int BN, int MODE>
+__device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, int m, int M,
+                                              int n0, int split, uint8_t* stage, int lane) {
+  const bool ok = m < M;
+  if constexpr (MODE == GEMM_BIAS_F32 || MODE == GEMM_BIAS_SILU_BF16 ||
+                MODE == GEMM_PARTIAL_F32) {
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      float v[32];
+      tmem_ld32(trow + c, v);
+      if constexpr (MODE == GEMM_PARTIAL_F32) {
+        uint4 u[8];
+        pack_f32x32(v, u);
+        float* dst = ok ? (float*)ep.out + split * ep.split_stride + (size_t)m * ep.ldo + n0 + c
+                        : nullptr;
+        warp_store_rows<128>(stage, u, dst, lane);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          v[i] += __ldg(ep.bias + n0 + c + i);
+          if constexpr (MODE == GEMM_BIAS_SILU_BF16) v[i] = silu_f(v[i]);
+        }
+        if constexpr (MODE == GEMM_BIAS_F32) {
+          uint4 u[8];
+          pack_f32x32(v, u);
+          warp_store_rows<128>(stage, u, ok ? (float*)ep.out + (size_t)m * ep.ldo + n0 + c : nullptr,
+                               lane);
+        } else {
+          uint4 u[4];
+          pack_bf16x32(v, u);
+          warp_store_rows<64>(stage, u, ok ? (bf16*)ep.out + (size_t)m * ep.ldo + n0 + c : nullptr,
+                              lane);
+        }
+      }
+    }
+  } else if constexpr (MODE == GEMM_GEGLU) {
+    // Tile columns [0, BN/2) hold gate rows n0/2 + c, [BN/2, BN) the matching up rows.
+    constexpr int half = BN / 2;
+#pragma unroll 1
+    for (int c = 0; c < half; c += 32) {
+      float g[32], u[32];
+      tmem_ld32(trow + c, g);
+      tmem_ld32(trow + half + c, u);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) g[i] = gelu_tanh_f(g[i]) * u[i];
+      uint4 pk[4];
+      pack_bf16x32(g, pk);
+      warp_store_rows<64>(stage, pk, ok ? (bf16*)ep.out + (size_t)m * ep.ldo + n0 / 2 + c : nullptr,
+                          lane);
+    }
+  } else if constexpr (MODE == GEMM_QKV_ROPE) {
+    // Weight rows are permuted so that tile column c < BN/2 holds head dim
+    // d = tj*BN/2 + c of segment `seg` and column c + BN/2 holds its rotate-half
+    // partner d + dh/2.  Segments: q heads 0..nq-1, then k, then v.
+    constexpr int half = BN / 2;
+    const int dh = ep.dh, seg = n0 / dh, tj = (n0 % dh) / BN;
+    int r = 0, t = 0, pos = 0;
+    if (ok) {
+      r = m / ep.T;
+      t = m - r * ep.T;
+      pos = __ldg(ep.prefix_len + r) + t;
+    }
+    bf16* dst;
+    if (seg < ep.nq)
+      dst = (bf16*)ep.q + (size_t)m * ep.nq * dh + seg * dh;
+    else
+      dst = (bf16*)(seg == ep.nq ? ep.kc : ep.vc) + ((size_t)r * ep.S_cap + pos) * dh;
+    const bool rotate = seg <= ep.nq;
+    const float4* cs4 = reinterpret_cast<const float4*>(ep.rope + (size_t)pos * (dh / 2) +
+                                                        tj * half);  // (cos, sin) pairs
+#pragma unroll 1
+    for (int c = 0; c < half; c += 32) {
+      float4 cs[16];
+      if (ok && rotate) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) cs[i] = __ldg(cs4 + c / 2 + i);
+      }
+      float x1[32], x2[32];
+      tmem_ld32(trow + c, x1);
+      tmem_ld32(trow + half + c, x2);
+      const int d0 = tj * half + c;
+      if (ok && rotate) {
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          const float a0 = x1[i], b0 = x2[i], a1 = x1[i + 1], b1 = x2[i + 1];
+          x1[i] = a0 * cs[i / 2].x - b0 * cs[i / 2].y;
+          x2[i] = b0 * cs[i / 2].x + a0 * cs[i / 2].y;
+          x1[i + 1] = a1 * cs[i / 2].z - b1 * cs[i / 2].w;
+          x2[i + 1] = b1 * cs[i / 2].z + a1 * cs[i / 2].w;
+        }
+      }
+      uint4 p1[4], p2[4];
+      pack_bf16x32(x1, p1);
+      pack_bf16x32(x2, p2);
+      warp_store_rows<64>(stage, p1, ok ? dst + d0 : nullptr, lane);
+      warp_store_rows<64>(stage, p2, ok ? dst + d0 + dh / 2 : nullptr, lane);
+    }
+  }
+}
+
+}  // namespace fva
