@@ -34,8 +34,19 @@ Readings where the paper is silent (the CUDA library takes the same ones):
 * R8 rotate-half RoPE with theta from the config at absolute position P_r + t;
   the prefix keys arrive already rotated; theta = 0 disables RoPE.
 * R9 gated MLP with tanh-approximate GELU on the gate branch.
+* R10 cold start (§3.2 "Cold start", Algorithm 1): a request whose buffer holds
+  n_valid < K real chunks keeps them in the noisiest slots K-n_valid .. K-1 and
+  padding in the cleaner slots; padding tokens are never keys, and their outputs
+  (velocity, emitted chunk, buffer slots) are meaningless.  A query with no
+  visible key at all (a padding token of a request without prefix) gets a zero
+  attention output.
+* R11 the queue has a fixed length: PushBack evicts the front slot during cold
+  start too, so a chunk receives exactly K updates between entering at the tail
+  and being emitted.
 * R12 the tail chunk z is either passed in or drawn from Philox4x32-10 +
   Box-Muller (``philox_normal_tail``).
+* Mask variants: "chunk_causal" (§3.1, the method) and "block_diagonal" (each
+  chunk sees the prefix and itself only: the no-causal ablation of §4).
 * R13 expert projections have no bias; in/out projections, time MLP and FiLM do.
 
 Parity: pinned by the tests in tests/test_oracle_pins.py (K=1 reduction to a
@@ -121,14 +132,19 @@ def chunk_of_token(n_tokens: int, chunk_tokens: int) -> np.ndarray:
     return np.arange(n_tokens) // chunk_tokens
 
 
-def visible_keys(prefix_len: int, chunk: int, chunk_tokens: int) -> Tuple[np.ndarray, np.ndarray]:
+def visible_keys(prefix_len: int, chunk: int, chunk_tokens: int, first_real: int = 0,
+                 mask: str = "chunk_causal") -> Tuple[np.ndarray, np.ndarray]:
     """Explicit key index lists seen by every token of chunk ``chunk`` (§3.1, R3).
 
     Returns (prefix indices, action-token indices): the whole prefix, and every
-    action token s of chunk c(s) <= chunk (own chunk bidirectional, earlier
-    chunks fully, later chunks never).
+    action token s with first_real <= c(s) <= chunk (own chunk bidirectional,
+    earlier real chunks fully, later chunks and padding never; R10).  With
+    mask="block_diagonal" only the chunk's own tokens (if it is real).
     """
-    return np.arange(prefix_len), np.arange((chunk + 1) * chunk_tokens)
+    lo = chunk if mask == "block_diagonal" else first_real
+    lo = max(lo, first_real)
+    hi = chunk + 1
+    return np.arange(prefix_len), np.arange(lo * chunk_tokens, max(lo, hi) * chunk_tokens)
 
 
 def key_limit_table(prefix_len: int, n_chunks: int, chunk_tokens: int) -> np.ndarray:
@@ -140,18 +156,23 @@ def key_limit_table(prefix_len: int, n_chunks: int, chunk_tokens: int) -> np.nda
 
 def chunk_causal_attention(q: np.ndarray, k_pre: np.ndarray, v_pre: np.ndarray,
                            k_act: np.ndarray, v_act: np.ndarray, chunk_tokens: int,
-                           scale: float) -> np.ndarray:
-    """MQA over unmasked keys only (R3, R4).
+                           scale: float, first_real: int = 0,
+                           mask: str = "chunk_causal") -> np.ndarray:
+    """MQA over unmasked keys only (R3, R4, R10).
 
     q [T, nq, dh]; k_pre/v_pre [P, dh]; k_act/v_act [T, dh] -> o [T, nq, dh].
     Each chunk's rows gather their visible keys by index and take an ordinary
-    softmax over exactly those keys: masked keys never enter the sum.
+    softmax over exactly those keys: masked keys never enter the sum.  Chunks
+    before ``first_real`` are padding (never keys); rows without any visible key
+    get zeros.
     """
     T = q.shape[0]
     o = np.zeros_like(q, dtype=f64)
     for c in range(T // chunk_tokens):
         rows = slice(c * chunk_tokens, (c + 1) * chunk_tokens)
-        ip, ia = visible_keys(k_pre.shape[0], c, chunk_tokens)
+        ip, ia = visible_keys(k_pre.shape[0], c, chunk_tokens, first_real, mask)
+        if ip.size + ia.size == 0:
+            continue
         keys = np.concatenate([k_pre[ip], k_act[ia]], axis=0)          # [S, dh]
         vals = np.concatenate([v_pre[ip], v_act[ia]], axis=0)
         qr = q[rows].reshape(-1, q.shape[-1])                          # [H*nq, dh]
@@ -186,15 +207,21 @@ def film(cond: np.ndarray, w, b, parts: int) -> List[np.ndarray]:
 
 def expert_velocity(weights: Dict, cfg: Dict, x: np.ndarray, tau: np.ndarray,
                     prefix_k: np.ndarray, prefix_v: np.ndarray,
-                    trace: Optional[Dict] = None, trace_layer: int = -1) -> np.ndarray:
+                    trace: Optional[Dict] = None, trace_layer: int = -1,
+                    n_valid: Optional[int] = None) -> np.ndarray:
     """One forward pass of the flow-matching action expert over one request's buffer.
 
     x [K, H, A] (slot 0 cleanest), tau [K], prefix_k/v [L, P, dh] (already rotated).
     Returns the velocity v [K, H, A] (fp64).  If ``trace`` is a dict, the inputs and
     outputs of every sub-step of layer ``trace_layer`` are stored in it.
+    n_valid (R10): real chunks in slots K-n_valid .. K-1, padding before them
+    (None: all K real).  cfg["mask"] selects the mask variant (default
+    "chunk_causal").
     """
     K, H, A = x.shape
     T = K * H
+    first_real = 0 if n_valid is None else K - int(n_valid)
+    mask = cfg.get("mask", "chunk_causal")
     W, nq, dh = cfg["width"], cfg["n_q_heads"], cfg["head_dim"]
     eps = cfg["rms_eps"]
     P = prefix_k.shape[1]
@@ -213,7 +240,7 @@ def expert_velocity(weights: Dict, cfg: Dict, x: np.ndarray, tau: np.ndarray,
         q = rope(q, pos, cfg["rope_theta"])
         k = rope(k, pos, cfg["rope_theta"])
         o = chunk_causal_attention(q, _w(prefix_k[l]), _w(prefix_v[l]), k, v, H,
-                                   1.0 / math.sqrt(dh))
+                                   1.0 / math.sqrt(dh), first_real, mask)
         h_mid = h + g1[c_tok] * (o.reshape(T, nq * dh) @ _w(lw["w_o"]).T)
         y2 = rms_norm(h_mid, eps) * (1.0 + s2[c_tok]) + b2[c_tok]
         m = gelu_tanh(y2 @ _w(lw["w_g"]).T) * (y2 @ _w(lw["w_u"]).T)
@@ -232,21 +259,26 @@ def expert_velocity(weights: Dict, cfg: Dict, x: np.ndarray, tau: np.ndarray,
 
 def stream_step(weights: Dict, cfg: Dict, buffer: np.ndarray, tau: np.ndarray,
                 prefix: Sequence[Tuple[np.ndarray, np.ndarray]],
-                fresh: np.ndarray) -> Tuple[np.ndarray, np.ndarray, np.ndarray]:
-    """One steady-streaming step (§3.2, Algorithm 1) for a batch of requests.
+                fresh: np.ndarray, n_valid: Optional[Sequence[int]] = None
+                ) -> Tuple[np.ndarray, np.ndarray, np.ndarray]:
+    """One streaming step (§3.2, Algorithm 1) for a batch of requests.
 
     buffer [B, K, H, A]; tau [B, K]; prefix[r] = (K_r, V_r) each [L, P_r, dh];
-    fresh [B, H, A] (the N(0, I) tail chunk).
+    fresh [B, H, A] (the N(0, I) tail chunk); n_valid [B] real chunks per request
+    (None: all K, steady streaming; fewer: a cold-start step, R10/R11).
     Returns (out [B, H, A], new buffer [B, K, H, A], velocity [B, K, H, A]), fp64.
 
     Per request: advance every chunk one level (x_k += Delta t_k v_k), pop the
     head chunk (now at tau_0 = 0) as the executable chunk, shift slots k+1 -> k,
-    push ``fresh`` into the tail slot.
+    push ``fresh`` into the tail slot.  In a cold-start step the popped chunk is
+    padding (the caller executes its default action instead).
     """
     B = buffer.shape[0]
     outs, news, vels = [], [], []
     for r in range(B):
-        vel = expert_velocity(weights, cfg, buffer[r], tau[r], prefix[r][0], prefix[r][1])
+        nv = None if n_valid is None else int(n_valid[r])
+        vel = expert_velocity(weights, cfg, buffer[r], tau[r], prefix[r][0], prefix[r][1],
+                              n_valid=nv)
         dt = delta_t(tau[r])
         adv = _w(buffer[r]) + dt[:, None, None] * vel
         outs.append(adv[0])

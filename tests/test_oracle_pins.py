@@ -338,3 +338,134 @@ def test_philox_tail_statistics():
 def test_key_limits_and_chunks():
     np.testing.assert_array_equal(O.chunk_of_token(6, 2), [0, 0, 1, 1, 2, 2])
     np.testing.assert_array_equal(O.key_limit_table(10, 3, 2), [12, 12, 14, 14, 16, 16])
+
+
+# ---------------------------------------------------------------------------
+# 8. cold start (§3.2 "Cold start", Algorithm 1; readings R10, R11)
+# ---------------------------------------------------------------------------
+
+def test_cold_start_all_valid_is_the_steady_step():
+    wl = tiny_wl(n_chunks=3, batch=2, prefix_lens=[5, 2])
+    w, pre, buf, tau = setup(wl)
+    fresh = WL.make_fresh_noise(wl, 1)[0]
+    a = O.stream_step(w, wl.as_config(), buf, tau, pre, fresh)
+    b = O.stream_step(w, wl.as_config(), buf, tau, pre, fresh, n_valid=[3, 3])
+    for x, y in zip(a, b):
+        np.testing.assert_array_equal(x, y)
+
+
+@pytest.mark.parametrize("n_valid", [1, 2, 3])
+def test_cold_start_padding_is_invisible(n_valid):
+    """Real chunks do not depend on the padding slots' contents or noise levels."""
+    K = 4
+    wl = tiny_wl(n_chunks=K)
+    w, pre, buf, tau = setup(wl)
+    cfg = wl.as_config()
+    c0 = K - n_valid
+    v0 = O.expert_velocity(w, cfg, buf[0], tau[0], pre[0][0], pre[0][1], n_valid=n_valid)
+    rng = np.random.default_rng(11)
+    buf2, tau2 = buf.copy(), tau.copy()
+    buf2[0, :c0] = 5 * rng.standard_normal(buf2[0, :c0].shape)
+    tau2[0, :c0] = np.sort(rng.uniform(0.001, tau[0, c0], size=c0))
+    v1 = O.expert_velocity(w, cfg, buf2[0], tau2[0], pre[0][0], pre[0][1], n_valid=n_valid)
+    np.testing.assert_array_equal(v0[c0:], v1[c0:])
+    # without the padding mask the same perturbation does reach the real chunks
+    if c0 > 0:
+        w0 = O.expert_velocity(w, cfg, buf[0], tau[0], pre[0][0], pre[0][1])
+        w1 = O.expert_velocity(w, cfg, buf2[0], tau2[0], pre[0][0], pre[0][1])
+        assert not np.allclose(w0[c0:], w1[c0:])
+
+
+@pytest.mark.parametrize("n_valid", [1, 2, 3])
+def test_cold_start_equals_shorter_buffer_without_rope(n_valid):
+    """Without RoPE positions do not matter, so the real chunks of a cold-start
+    buffer move exactly like a K = n_valid buffer holding only them."""
+    K = 4
+    wl = tiny_wl(n_chunks=K, rope_theta=0.0)
+    w, pre, buf, tau = setup(wl)
+    cfg = wl.as_config()
+    c0 = K - n_valid
+    full = O.expert_velocity(w, cfg, buf[0], tau[0], pre[0][0], pre[0][1], n_valid=n_valid)
+    short = O.expert_velocity(w, cfg, buf[0, c0:], tau[0, c0:], pre[0][0], pre[0][1])
+    np.testing.assert_allclose(full[c0:], short, rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("P,H,K,nq,dh,first_real,mask",
+                         [(3, 2, 3, 2, 4, 1, "chunk_causal"), (0, 3, 3, 1, 4, 2, "chunk_causal"),
+                          (2, 2, 3, 2, 4, 0, "block_diagonal"),
+                          (0, 2, 4, 1, 6, 1, "block_diagonal")])
+def test_masked_attention_brute_force(P, H, K, nq, dh, first_real, mask):
+    """Padding and mask variants against an explicit per-pair predicate; rows with
+    no visible key give zeros (R10)."""
+    rng = np.random.default_rng(P + 10 * H + 100 * K + first_real)
+    T = H * K
+    q = rng.standard_normal((T, nq, dh))
+    kp, vp = rng.standard_normal((P, dh)), rng.standard_normal((P, dh))
+    ka, va = rng.standard_normal((T, dh)), rng.standard_normal((T, dh))
+    scale = 1 / math.sqrt(dh)
+    got = O.chunk_causal_attention(q, kp, vp, ka, va, H, scale, first_real, mask)
+
+    def visible(t, s):
+        if s < P:
+            return True
+        cs, ct = (s - P) // H, t // H
+        if cs < first_real:
+            return False
+        return cs == ct if mask == "block_diagonal" else cs <= ct
+
+    for t in range(T):
+        for hh in range(nq):
+            idx = [s for s in range(P + T) if visible(t, s)]
+            if not idx:
+                assert np.all(got[t, hh] == 0)
+                continue
+            keys = [kp[s] if s < P else ka[s - P] for s in idx]
+            vals = [vp[s] if s < P else va[s - P] for s in idx]
+            logits = [sum(q[t, hh, d] * kk[d] for d in range(dh)) * scale for kk in keys]
+            mx = max(logits)
+            ex = [math.exp(z - mx) for z in logits]
+            ref = [sum(e * vv[d] for e, vv in zip(ex, vals)) / sum(ex) for d in range(dh)]
+            np.testing.assert_allclose(got[t, hh], ref, rtol=1e-12, atol=1e-12)
+
+
+def test_cold_start_episode_constant_velocity():
+    """Algorithm 1 from an empty buffer: K-1 cold-start steps with n_valid = 1..K-1,
+    then steady streaming.  The first sample z_0 is emitted at step K after exactly
+    K updates (R11), i.e. as z_0 - b when tau_K = 1; every later tail likewise."""
+    K = 4
+    wl = tiny_wl(n_chunks=K)
+    w, pre, _, tau = setup(wl)
+    b = np.linspace(0.25, -0.75, wl.action_dim)
+    z = zero_expert(w, b)
+    S = 3 * K
+    noise = WL.make_fresh_noise(wl, S + 1)
+    state = np.zeros((1, K, wl.chunk_tokens, wl.action_dim))
+    state[0, -1] = noise[0][0]                      # [pad, ..., pad, z_0]
+    emitted = []
+    for s in range(S):
+        nv = [min(K, s + 1)]
+        out, state, _ = O.stream_step(z, wl.as_config(), state, tau, pre, noise[s + 1], n_valid=nv)
+        emitted.append(out)
+    np.testing.assert_allclose(emitted[K - 1][0], noise[0][0] - b, atol=1e-12)
+    for s in range(K, S):
+        np.testing.assert_allclose(emitted[s][0], noise[s - K + 1][0] - b, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# 9. the no-causal (block-diagonal) ablation mask
+# ---------------------------------------------------------------------------
+
+def test_block_diagonal_chunks_are_independent_without_rope():
+    """With the block-diagonal mask and no RoPE every chunk moves exactly like a
+    K = 1 buffer holding it alone; with the chunk-causal mask it does not."""
+    K = 3
+    wl = tiny_wl(n_chunks=K, rope_theta=0.0)
+    w, pre, buf, tau = setup(wl)
+    cfg = dict(wl.as_config(), mask="block_diagonal")
+    full = O.expert_velocity(w, cfg, buf[0], tau[0], pre[0][0], pre[0][1])
+    for c in range(K):
+        alone = O.expert_velocity(w, cfg, buf[0, c:c + 1], tau[0, c:c + 1], pre[0][0], pre[0][1])
+        np.testing.assert_allclose(full[c], alone[0], rtol=1e-12, atol=1e-12)
+    causal = O.expert_velocity(w, wl.as_config(), buf[0], tau[0], pre[0][0], pre[0][1])
+    np.testing.assert_array_equal(causal[0], full[0])   # chunk 0 sees only itself either way
+    assert not np.allclose(causal[1:], full[1:])
