@@ -56,6 +56,10 @@ typedef enum fva_dtype {
 
 /* fva_config.flags */
 #define FVA_FLAG_NO_GRAPH 1u  /* launch the step kernel by kernel instead of replaying a CUDA graph */
+/* Block-diagonal mask: every chunk attends to the prefix and to itself only (the
+ * no-causal ablation of the paper's Sec. 4) instead of the chunk-causal mask of
+ * Sec. 3.1. */
+#define FVA_FLAG_BLOCK_DIAGONAL 2u
 
 /*
  * Shape and numerics of the action expert and of the streaming buffer.
@@ -184,10 +188,25 @@ typedef struct fva_step_opts {
   int32_t trace_layer;       /* >= 0: write that layer's intermediates to trace_out            */
   int32_t reserved;
   float* trace_out;          /* device fp32, fva_trace_floats(h, batch) floats; see below      */
+  const int32_t* n_valid;    /* host int32 [batch], each in 1..K: real chunks per request      */
 } fva_step_opts;
 
 /*
- * fva_step with options.  With trace_layer >= 0 the step runs kernel by kernel
+ * fva_step with options.
+ *
+ * Cold start (Sec. 3.2, Algorithm 1): with n_valid set, request r holds n_valid[r]
+ * real chunks in slots K - n_valid[r] .. K-1 and padding in the cleaner slots
+ * before them.  Padding tokens are never attention keys, so the real chunks
+ * move as if the padding were absent; the padding slots' velocities, the
+ * emitted chunk while it is padding and the padding slots of the updated buffer
+ * are meaningless (the caller executes its default action instead).  The roll
+ * and the tail push are those of a steady step (the queue keeps its length), so
+ * Algorithm 1 is: buffer = [pad, ..., pad, z]; K-1 steps with n_valid = 1 .. K-1;
+ * then steady steps (n_valid NULL or K).  A query without any visible key (a
+ * padding token of a request with no prefix) gets a zero attention output.
+ * INVALID_ARG if an entry is outside 1..K.
+ *
+ * With trace_layer >= 0 the step runs kernel by kernel
  * (no graph) and, for M = batch*K*H rows, writes fp32 copies of that layer's
  * tensors to trace_out back to back in this order:
  *   h_in [M, W], y1 [M, W], q [M, nq dh] (after RoPE), k [M, dh] (after RoPE),

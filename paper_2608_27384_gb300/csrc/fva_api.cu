@@ -187,6 +187,8 @@ struct fva_handle {
   uint64_t use_clock = 0;
 
   float* tau_dev() const { return params_dev; }
+  // padding tokens (K - n_valid) * H per request of the current step
+  int* pad_dev() const { return reinterpret_cast<int*>(params_dev + 2 * BKmax + 2); }
   float* dt_dev() const { return params_dev + BKmax; }
   unsigned long long* step_dev() const {
     return reinterpret_cast<unsigned long long*>(params_dev + 2 * BKmax);
@@ -257,6 +259,8 @@ fva_status validate_config(const fva_config* c) {
       !std::isfinite(c->rope_theta))
     return fail(FVA_ERR_INVALID_ARG, "bad rms_eps / rope_theta / timestep periods");
   if (c->action_dim > 128) return fail(FVA_ERR_UNSUPPORTED, "action_dim > 128");
+  if (c->flags & ~(FVA_FLAG_NO_GRAPH | FVA_FLAG_BLOCK_DIAGONAL))
+    return fail(FVA_ERR_INVALID_ARG, "unknown flags 0x%x", c->flags);
   const long long T = (long long)c->n_chunks * c->chunk_tokens;
   if (T * c->max_batch > (1LL << 24) || c->max_prefix > (1 << 20) || c->n_layers > 1024)
     return fail(FVA_ERR_UNSUPPORTED, "sizes too large");
@@ -441,7 +445,7 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
         (st = dalloc(h, &h->att_part_ml, tiles * h->attn_max_splits * 128)))
       return st;
   }
-  h->params_floats = 2 * h->BKmax + 2;
+  h->params_floats = 2 * h->BKmax + 2 + h->Bmax;
   if ((st = dalloc(h, &h->params_dev, h->params_floats))) return st;
   CUDA_TRY(cudaMallocHost((void**)&h->params_host,
                           sizeof(float) * h->params_floats * FVA_PARAM_RING));
@@ -973,6 +977,8 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       aa.kv_row0 = l * h->Bmax * h->S_cap;
       aa.scale_log2 = 1.4426950408889634f / std::sqrt((float)h->dh);
       aa.err = h->err_dev;
+      aa.pad_tokens = h->pad_dev();
+      aa.block_diag = (h->cfg.flags & FVA_FLAG_BLOCK_DIAGONAL) ? 1 : 0;
       mark(FVA_K_ATTENTION, l);
       CUDA_TRY(launch_tc_attention(&h->m_q, &h->m_k, &h->m_v, aa, B, s));
       if (aa.max_splits > 1) {
@@ -981,6 +987,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       }
     } else {
       launch_f32_attention((float*)h->q, (float*)kc_l, (float*)vc_l, h->prefix_len_dev,
+                           h->pad_dev(), (h->cfg.flags & FVA_FLAG_BLOCK_DIAGONAL) ? 1 : 0,
                            (float*)h->attn, B, h->T, h->H, h->nq, h->dh, h->S_cap, h->S_cap, s);
     }
     if (trace) launch_to_f32(h->attn, bf, tr_at(o_att), (long long)M * Dq, s);
@@ -1170,6 +1177,11 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     return fail(FVA_ERR_INVALID_ARG, "trace_layer %d >= n_layers", opts->trace_layer);
   if (opts && opts->trace_layer >= 0 && !opts->trace_out)
     return fail(FVA_ERR_INVALID_ARG, "trace_out is NULL");
+  if (opts && opts->n_valid)
+    for (int r = 0; r < batch; ++r)
+      if (opts->n_valid[r] < 1 || opts->n_valid[r] > h->K)
+        return fail(FVA_ERR_INVALID_ARG, "n_valid[%d] = %d outside [1, %d]", r,
+                    opts->n_valid[r], h->K);
   for (int r = 0; r < batch; ++r) {
     float prev = 0.f;
     for (int k = 0; k < h->K; ++k) {
@@ -1210,6 +1222,9 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     }
   const unsigned long long step = h->step_index++;
   std::memcpy(ph + 2 * h->BKmax, &step, sizeof(step));
+  int* pad = reinterpret_cast<int*>(ph + 2 * h->BKmax + 2);
+  for (int r = 0; r < h->Bmax; ++r)
+    pad[r] = (opts && opts->n_valid && r < batch) ? (h->K - opts->n_valid[r]) * h->H : 0;
   CUDA_TRY(cudaMemcpyAsync(h->params_dev, ph, sizeof(float) * h->params_floats,
                            cudaMemcpyHostToDevice, s));
   CUDA_TRY(cudaEventRecord(h->ring_ev[slot], s));

@@ -138,6 +138,11 @@ struct AttnArgs {
   int kv_row0;          // first KV row of this layer in the 2D view
   float scale_log2;     // log2(e) / sqrt(dh)
   int* err;
+  // Action keys a row sees start at P + lo: lo = pad_tokens[r] (cold-start
+  // padding; nullptr = 0), and under the block-diagonal mask at least the row's
+  // own chunk start.
+  const int* pad_tokens;
+  int block_diag;
 };
 
 constexpr int kAttnKeysPerSplit = 256;
@@ -226,7 +231,8 @@ void launch_f32_qkv_rope(const float* C, float* q, float* kc, float* vc,
                          int nq, int dh, cudaStream_t s);
 void launch_f32_geglu(const float* C, float* out, int M, int F, cudaStream_t s);
 void launch_f32_attention(const float* q, const float* kc, const float* vc,
-                          const int* prefix_len, float* out, int B, int T, int H, int nq,
-                          int dh, int S_cap, int max_keys, cudaStream_t s);
+                          const int* prefix_len, const int* pad_tokens, int block_diag,
+                          float* out, int B, int T, int H, int nq, int dh, int S_cap,
+                          int max_keys, cudaStream_t s);
 
 }  // namespace fva

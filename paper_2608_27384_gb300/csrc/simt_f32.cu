@@ -132,8 +132,10 @@ void launch_f32_geglu(const float* C, float* out, int M, int F, cudaStream_t s) 
 // One CTA per (token row, head): softmax over the row's visible keys only.
 __global__ void f32_attention_kernel(const float* __restrict__ q, const float* __restrict__ kc,
                                      const float* __restrict__ vc,
-                                     const int* __restrict__ prefix_len, float* __restrict__ out,
-                                     int T, int H, int nq, int dh, int S_cap) {
+                                     const int* __restrict__ prefix_len,
+                                     const int* __restrict__ pad_tokens, int block_diag,
+                                     float* __restrict__ out, int T, int H, int nq, int dh,
+                                     int S_cap) {
   extern __shared__ float sm[];  // [dh] query, then [limit] scores
   const int m = blockIdx.x, head = blockIdx.y;
   const int r = m / T, t = m % T;
@@ -141,6 +143,9 @@ __global__ void f32_attention_kernel(const float* __restrict__ q, const float* _
   pdl_wait();
   const int P = prefix_len[r];
   const int limit = attn_key_limit(P, t, H);
+  // action keys below P + lo are padding (cold start) or, block-diagonal, other chunks
+  const int pad = pad_tokens ? pad_tokens[r] : 0;
+  const int lo = P + (block_diag ? max(pad, (t / H) * H) : pad);
   float* sq = sm;
   float* sc = sm + dh;
   const float* qrow = q + ((size_t)m * nq + head) * dh;
@@ -152,7 +157,7 @@ __global__ void f32_attention_kernel(const float* __restrict__ q, const float* _
   for (int s = threadIdx.x; s < limit; s += blockDim.x) {
     float acc = 0.f;
     for (int d = 0; d < dh; ++d) acc = fmaf(sq[d], K[(size_t)s * dh + d], acc);
-    sc[s] = acc * scale;
+    sc[s] = (s < P || s >= lo) ? acc * scale : -INFINITY;
   }
   __syncthreads();
   __shared__ float red[32];
@@ -166,7 +171,7 @@ __global__ void f32_attention_kernel(const float* __restrict__ q, const float* _
   __syncthreads();
   float sum = 0.f;
   for (int s = threadIdx.x; s < limit; s += blockDim.x) {
-    const float p = expf(sc[s] - mx);
+    const float p = mx > -INFINITY ? expf(sc[s] - mx) : 0.f;  // no visible key: zeros
     sc[s] = p;
     sum += p;
   }
@@ -175,7 +180,7 @@ __global__ void f32_attention_kernel(const float* __restrict__ q, const float* _
   __syncthreads();
   sum = 0.f;
   for (int w = 0; w < (int)(blockDim.x >> 5); ++w) sum += red[w];
-  const float inv = 1.f / sum;
+  const float inv = sum > 0.f ? 1.f / sum : 0.f;
   float* orow = out + ((size_t)m * nq + head) * dh;
   for (int d = threadIdx.x; d < dh; d += blockDim.x) {
     float acc = 0.f;
@@ -185,13 +190,14 @@ __global__ void f32_attention_kernel(const float* __restrict__ q, const float* _
 }
 
 void launch_f32_attention(const float* q, const float* kc, const float* vc,
-                          const int* prefix_len, float* out, int B, int T, int H, int nq,
-                          int dh, int S_cap, int max_keys, cudaStream_t s) {
+                          const int* prefix_len, const int* pad_tokens, int block_diag,
+                          float* out, int B, int T, int H, int nq, int dh, int S_cap,
+                          int max_keys, cudaStream_t s) {
   if (B * T <= 0) return;
   dim3 grid(B * T, nq);
   const size_t smem = sizeof(float) * (dh + max_keys);
-  launch_pdl(f32_attention_kernel, grid, dim3(128), smem, s, q, kc, vc, prefix_len, out, T, H,
-             nq, dh, S_cap);
+  launch_pdl(f32_attention_kernel, grid, dim3(128), smem, s, q, kc, vc, prefix_len, pad_tokens,
+             block_diag, out, T, H, nq, dh, S_cap);
 }
 
 }  // namespace fva

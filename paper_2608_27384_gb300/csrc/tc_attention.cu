@@ -192,6 +192,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int t = t0 + row / a.nq;
     const bool valid = t < a.T;
     const int limit = valid ? attn_key_limit(P, t, a.H) : 0;
+    // action keys in [P, P + lo) are padding (cold start) or, under the
+    // block-diagonal mask, earlier chunks
+    const int pad = a.pad_tokens ? __ldg(a.pad_tokens + r) : 0;
+    const int lo = a.block_diag && valid ? max(pad, (t / a.H) * a.H) : pad;
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
     const bool has_blk = g < nblk;
     const int key0 = (kb0 + g) * kKB;
@@ -202,6 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     float mx = -INFINITY, l = 0.f;
     const int nvis = min(kKB, max(0, limit - key0));
+    const int p_rel = P - key0, lo_rel = P + lo - key0;  // hidden: p_rel <= i < lo_rel
     uint4 pk[8];  // P of this block against the block's own max, bf16, logical order
     if (good && has_blk) {
       uint32_t sv[64];
@@ -212,7 +217,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld_wait();
 #pragma unroll
       for (int i = 0; i < 64; ++i)
-        if (i < nvis) mx = fmaxf(mx, __uint_as_float(sv[i]));
+        if (i < nvis && (i < p_rel || i >= lo_rel)) mx = fmaxf(mx, __uint_as_float(sv[i]));
       const float mscaled = mx > -INFINITY ? mx * a.scale_log2 : 0.f;
 #pragma unroll
       for (int c = 0; c < 8; ++c) {  // keys 8c .. 8c+7
@@ -221,7 +226,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < 8; ++i) {
           const int kk = c * 8 + i;
           const float e = exp2f(fmaf(__uint_as_float(sv[kk]), a.scale_log2, -mscaled));
-          const float pr = kk < nvis ? __bfloat162float(__float2bfloat16_rn(e)) : 0.f;
+          const bool vis = kk < nvis && (kk < p_rel || kk >= lo_rel);
+          const float pr = vis ? __bfloat162float(__float2bfloat16_rn(e)) : 0.f;
           l += pr;
           p[i] = pr;
         }
@@ -331,7 +337,8 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
   float m_all = warp_max(ml.y > 0.f ? ml.x : -INFINITY);
   // each split stored O_s / l_s; its weight is 2^((m_s - m) c) l_s
   const float w = ml.y > 0.f ? exp2f((ml.x - m_all) * a.scale_log2) * ml.y : 0.f;
-  const float inv = 1.f / warp_sum(w);
+  const float tot = warp_sum(w);
+  const float inv = tot > 0.f ? 1.f / tot : 0.f;  // no visible key in any split: zeros
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   for (int s0 = 0; s0 < nsplit; s0 += 8) {  // up to 8 splits' loads in flight
     uint4 x[8];

@@ -10,8 +10,8 @@ from typing import Dict, List, Optional, Sequence, Tuple
 
 import numpy as np
 
-from . import (FVA_BF16, FVA_FP32, fva_create, fva_destroy, fva_load_weights,
-               fva_set_prefix_kv, make_config)
+from . import (FVA_BF16, FVA_FLAG_BLOCK_DIAGONAL, FVA_FP32, fva_create, fva_destroy,
+               fva_load_weights, fva_set_prefix_kv, make_config)
 
 
 def _bits(x: np.ndarray) -> np.ndarray:
@@ -26,6 +26,8 @@ def storage(arr: np.ndarray, bf16: bool) -> np.ndarray:
 def config_for(wl, max_batch: Optional[int] = None, max_prefix: Optional[int] = None,
                flags: int = 0, noise_seed: int = 0):
     bf16 = wl.dtype == "bf16"
+    if getattr(wl, "mask", "chunk_causal") == "block_diagonal":
+        flags |= FVA_FLAG_BLOCK_DIAGONAL
     return make_config(dtype=FVA_BF16 if bf16 else FVA_FP32, n_layers=wl.n_layers,
                        width=wl.width, n_q_heads=wl.n_q_heads, head_dim=wl.head_dim,
                        mlp_dim=wl.mlp_dim, action_dim=wl.action_dim, n_chunks=wl.n_chunks,

@@ -56,7 +56,8 @@ class Case:
     def dev(self, a):
         return self.torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
-    def run(self, buf=None, tau=None, fresh=None, want_vel=True, trace_layer=-1, batch=None):
+    def run(self, buf=None, tau=None, fresh=None, want_vel=True, trace_layer=-1, batch=None,
+            n_valid=None):
         """One GPU step.  Returns dict(out, buffer, vel[, trace]) as numpy arrays."""
         import paper_2608_27384_gb300 as fva
         torch = self.torch
@@ -73,7 +74,8 @@ class Case:
         if trace_layer >= 0:
             d_tr = torch.empty(fva.fva_trace_floats(self.handle, B), device="cuda")
         fva.fva_step_ex(self.handle, d_buf, tau[:B], d_out, B, fresh_noise=d_fresh,
-                        velocity_out=d_vel, trace_layer=trace_layer, trace_out=d_tr)
+                        velocity_out=d_vel, trace_layer=trace_layer, trace_out=d_tr,
+                        n_valid=None if n_valid is None else list(n_valid)[:B])
         torch.cuda.synchronize()
         res = dict(out=d_out.cpu().numpy(), buffer=d_buf.cpu().numpy())
         if want_vel:
@@ -82,7 +84,7 @@ class Case:
             res["trace"] = d_tr.cpu().numpy()
         return res
 
-    def oracle_step(self, buf=None, tau=None, fresh=None, batch=None):
+    def oracle_step(self, buf=None, tau=None, fresh=None, batch=None, n_valid=None):
         wl = self.wl
         B = batch or wl.batch
         buf = self.buf if buf is None else buf
@@ -90,7 +92,7 @@ class Case:
         if fresh is None:
             fresh = np.zeros((B, wl.chunk_tokens, wl.action_dim), np.float32)
         return oracle.stream_step(self.w, wl.as_config(), buf[:B], tau[:B], self.prefix[:B],
-                                  fresh[:B])
+                                  fresh[:B], None if n_valid is None else list(n_valid)[:B])
 
     def close(self):
         self.dec.close()

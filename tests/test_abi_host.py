@@ -50,10 +50,31 @@ def _cfg(fva, **over):
     return c
 
 
-def test_config_struct_layout(fva):
+def test_config_struct_layout(fva, tmp_path):
+    """The binding's ctypes structs have the C header's layout (compiled with gcc)."""
+    import shutil
+    import subprocess
     assert ctypes.sizeof(fva.fva_config) == 80
     assert fva.fva_config.noise_seed.offset == 72
-    assert ctypes.sizeof(fva.fva_step_opts) == 32
+    assert ctypes.sizeof(fva.fva_step_opts) == 40
+    assert fva.fva_step_opts.n_valid.offset == 32
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "layout.c"
+    src.write_text(
+        "#include <stdio.h>\n#include <stddef.h>\n#include \"fva.h\"\n"
+        "int main(void) { printf(\"%zu %zu %zu %zu %zu\\n\", sizeof(fva_config),"
+        " offsetof(fva_config, noise_seed), sizeof(fva_step_opts),"
+        " offsetof(fva_step_opts, trace_out), offsetof(fva_step_opts, n_valid)); return 0; }\n")
+    exe = tmp_path / "layout"
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.run([cc, "-I", inc, str(src), "-o", str(exe)], check=True)
+    got = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True,
+                                          check=True).stdout.split()]
+    assert got == [ctypes.sizeof(fva.fva_config), fva.fva_config.noise_seed.offset,
+                   ctypes.sizeof(fva.fva_step_opts), fva.fva_step_opts.trace_out.offset,
+                   fva.fva_step_opts.n_valid.offset]
 
 
 @pytest.mark.parametrize("field,value,status", [

@@ -1,0 +1,141 @@
+"""GPU parity of the cold-start steps (padding chunks, Algorithm 1) and of the
+block-diagonal mask variant, through the C ABI, against the CPU oracle.
+
+Only real chunks are compared: the velocity of slots K-n_valid .. K-1, the
+updated buffer slots they move into, and the emitted chunk once it is real.
+"""
+import numpy as np
+import pytest
+
+import workloads as WL
+from gpu_util import TOL, VEL_REL_L2, Case, assert_close
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2608_27384_gb300 as fva
+    fva.lib()
+    torch.cuda.set_device(0)
+
+
+def _workload(dtype, **over):
+    if dtype == "bf16":
+        base = dict(n_chunks=4, prefix_lens=[300])
+        base.update(over)
+        return WL.small_bf16_workload(**base)
+    wl = WL.standard_workloads()["tiny_fp32"]
+    d = dict(wl.__dict__)
+    d.update(dict(n_chunks=4, prefix_lens=[40]))
+    d.update(over)
+    return WL.Workload(**d)
+
+
+def check_real(res, ref, n_valid, K, dtype):
+    out_ref, new_ref, vel_ref = ref
+    tol = TOL[dtype]
+    for r, nv in enumerate(n_valid):
+        c0 = K - nv
+        assert np.all(np.isfinite(res["vel"][r, c0:]))
+        assert_close(res["vel"][r, c0:], vel_ref[r, c0:], rel_l2=VEL_REL_L2[dtype],
+                     what=f"velocity r={r} n_valid={nv}")
+        lo = max(0, c0 - 1)  # slot c moves to c - 1; the tail slot takes the fresh chunk
+        assert_close(res["buffer"][r, lo:], new_ref[r, lo:], what=f"buffer r={r}", **tol)
+        if nv == K:
+            assert_close(res["out"][r], out_ref[r], what=f"out r={r}", **tol)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+@pytest.mark.parametrize("n_valid", [[1], [2], [3], [4]])
+def test_cold_start_step(dtype, n_valid):
+    wl = _workload(dtype)
+    case = Case(wl)
+    try:
+        fresh = WL.make_fresh_noise(wl, 1)[0]
+        res = case.run(fresh=fresh, n_valid=n_valid)
+        check_real(res, case.oracle_step(fresh=fresh, n_valid=n_valid), n_valid, wl.n_chunks, dtype)
+    finally:
+        case.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_cold_start_ragged_batch(dtype):
+    """One launch, three requests at different cold-start stages and prefixes,
+    one of them without any prefix (its padding queries see no key at all)."""
+    prefixes = [0, 37, 280] if dtype == "bf16" else [0, 9, 40]
+    wl = _workload(dtype, batch=3, prefix_lens=prefixes, tau_mode="beta")
+    n_valid = [1, 3, 2]
+    case = Case(wl)
+    try:
+        fresh = WL.make_fresh_noise(wl, 1)[0]
+        res = case.run(fresh=fresh, n_valid=n_valid)
+        check_real(res, case.oracle_step(fresh=fresh, n_valid=n_valid), n_valid, wl.n_chunks, dtype)
+    finally:
+        case.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_padding_is_invisible_bitwise(dtype):
+    """Changing the padding slots' contents and noise levels leaves every real
+    chunk's velocity bit-identical on the GPU."""
+    wl = _workload(dtype)
+    K, nv = wl.n_chunks, 2
+    c0 = K - nv
+    case = Case(wl)
+    try:
+        a = case.run(n_valid=[nv])
+        rng = np.random.default_rng(5)
+        buf2, tau2 = case.buf.copy(), case.tau.copy()
+        buf2[0, :c0] = 4 * rng.standard_normal(buf2[0, :c0].shape).astype(np.float32)
+        tau2[0, :c0] = np.sort(rng.uniform(0.001, case.tau[0, c0], size=c0)).astype(np.float32)
+        b = case.run(buf=buf2, tau=tau2, n_valid=[nv])
+        np.testing.assert_array_equal(a["vel"][0, c0:], b["vel"][0, c0:])
+        c = case.run(buf=buf2, tau=tau2)          # without the padding mask it leaks
+        assert not np.array_equal(a["vel"][0, c0:], c["vel"][0, c0:])
+    finally:
+        case.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_cold_start_episode(dtype):
+    """Algorithm 1 from [pad, ..., pad, z_0]: K-1 cold-start steps with n_valid =
+    1 .. K-1, then steady steps; GPU and oracle run the same sequence with the
+    same injected tails, and every real chunk they emit agrees."""
+    wl = _workload(dtype, n_chunks=3)
+    K = wl.n_chunks
+    case = Case(wl)
+    try:
+        noise = WL.make_fresh_noise(wl, K + 3)
+        g = np.zeros_like(case.buf)
+        g[0, -1] = noise[0][0]
+        o = g.astype(np.float64)
+        for s in range(K + 2):
+            nv = [min(K, s + 1)]
+            res = case.run(buf=g, fresh=noise[s + 1], n_valid=nv)
+            out_ref, o, _ = case.oracle_step(buf=o, fresh=noise[s + 1], n_valid=nv)
+            g = res["buffer"]
+            real = max(0, K - nv[0] - 1)
+            assert_close(g[0, real:], o[0, real:], what=f"buffer step {s}", **TOL[dtype])
+            if nv[0] == K:
+                assert_close(res["out"], out_ref, what=f"emitted step {s}", **TOL[dtype])
+    finally:
+        case.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_block_diagonal_mask(dtype):
+    wl = _workload(dtype, mask="block_diagonal", n_chunks=3)
+    case = Case(wl)
+    try:
+        fresh = WL.make_fresh_noise(wl, 1)[0]
+        res = case.run(fresh=fresh)
+        out_ref, new_ref, vel_ref = case.oracle_step(fresh=fresh)
+        assert_close(res["out"], out_ref, what="out", **TOL[dtype])
+        assert_close(res["buffer"], new_ref, what="buffer", **TOL[dtype])
+        assert_close(res["vel"], vel_ref, rel_l2=VEL_REL_L2[dtype], what="velocity")
+    finally:
+        case.close()

@@ -56,6 +56,7 @@ class Workload:
     t_min_period: float = 4e-3
     t_max_period: float = 4.0
     seed: int = 0
+    mask: str = "chunk_causal"      # or "block_diagonal" (no-causal ablation)
 
     @property
     def tokens(self) -> int:
@@ -73,7 +74,7 @@ class Workload:
             action_dim=self.action_dim, n_chunks=self.n_chunks,
             chunk_tokens=self.chunk_tokens, rms_eps=self.rms_eps,
             rope_theta=self.rope_theta, t_min_period=self.t_min_period,
-            t_max_period=self.t_max_period)
+            t_max_period=self.t_max_period, mask=self.mask)
 
 
 def _serving_prefix_lens(n: int, lo: int, hi: int, seed: int) -> List[int]:
