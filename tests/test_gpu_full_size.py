@@ -20,7 +20,9 @@ def _cuda():
 
 @pytest.mark.parametrize("name,recipe", [("tiny_fp32", "paper"), ("pi05_2view", "paper"),
                                          ("pi05_2view", "unit_gate"), ("pi05_3view", "paper"),
-                                         ("serving16", "paper"), ("long_b4", "paper")])
+                                         ("serving16", "paper"), ("long_b4", "paper"),
+                                         ("libero_k4h10", "paper"), ("robotwin_k4h20", "paper"),
+                                         ("k5h10", "paper")])
 def test_full_size_workload(name, recipe):
     wl = WL.standard_workloads()[name]
     case = Case(wl, recipe=recipe)

@@ -83,7 +83,9 @@ def _serving_prefix_lens(n: int, lo: int, hi: int, seed: int) -> List[int]:
 
 
 def standard_workloads() -> Dict[str, Workload]:
-    """The five workloads of the hot-path study, by name."""
+    """The workloads of the hot-path study, by name: the five of the main study,
+    then the paper's own deployment buffer shapes (Sec. 4 and App. A.2: chunk size
+    10 / 20 with buffer length 4 / 5) on the same pi0.5-sized expert."""
     expert = dict(dtype=DTYPE_BF16, n_layers=18, width=1024, n_q_heads=8, head_dim=256,
                   mlp_dim=4096, action_dim=32, chunk_tokens=50)
     return {
@@ -99,6 +101,15 @@ def standard_workloads() -> Dict[str, Workload]:
                               tau_mode="beta", **expert),
         # Long buffer: K=20 x H=50 = 1000 action tokens, prefix 1024, batch 4.
         "long_b4": Workload("long_b4", n_chunks=20, batch=4, prefix_lens=[1024] * 4, **expert),
+        # LIBERO setting: chunk size 10, buffer length 4 (40 action tokens), 2 views.
+        "libero_k4h10": Workload("libero_k4h10", n_chunks=4, batch=1, prefix_lens=[560],
+                                 **dict(expert, chunk_tokens=10)),
+        # RoboTwin / real-robot setting: chunk size 20, buffer length 4, 3 views.
+        "robotwin_k4h20": Workload("robotwin_k4h20", n_chunks=4, batch=1, prefix_lens=[816],
+                                   **dict(expert, chunk_tokens=20)),
+        # SmolVLA setting's buffer: chunk size 10, buffer length 5, 2 views.
+        "k5h10": Workload("k5h10", n_chunks=5, batch=1, prefix_lens=[560],
+                          **dict(expert, chunk_tokens=10)),
     }
 
 
