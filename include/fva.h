@@ -57,7 +57,7 @@ typedef enum fva_dtype {
 /* fva_config.flags */
 #define FVA_FLAG_NO_GRAPH 1u  /* launch the step kernel by kernel instead of replaying a CUDA graph */
 /* Block-diagonal mask: every chunk attends to the prefix and to itself only (the
- * no-causal ablation of the paper's Sec. 4) instead of the chunk-causal mask of
+ * no-causal ablation of the paper's App. A.3) instead of the chunk-causal mask of
  * Sec. 3.1. */
 #define FVA_FLAG_BLOCK_DIAGONAL 2u
 

@@ -46,7 +46,7 @@ Readings where the paper is silent (the CUDA library takes the same ones):
 * R12 the tail chunk z is either passed in or drawn from Philox4x32-10 +
   Box-Muller (``philox_normal_tail``).
 * Mask variants: "chunk_causal" (§3.1, the method) and "block_diagonal" (each
-  chunk sees the prefix and itself only: the no-causal ablation of §4).
+  chunk sees the prefix and itself only: the no-causal ablation of App. A.3).
 * R13 expert projections have no bias; in/out projections, time MLP and FiLM do.
 
 Parity: pinned by the tests in tests/test_oracle_pins.py (K=1 reduction to a

@@ -84,7 +84,7 @@ def _serving_prefix_lens(n: int, lo: int, hi: int, seed: int) -> List[int]:
 
 def standard_workloads() -> Dict[str, Workload]:
     """The workloads of the hot-path study, by name: the five of the main study,
-    then the paper's own deployment buffer shapes (Sec. 4 and App. A.2: chunk size
+    then the paper's own deployment buffer shapes (App. A.1 and A.2: chunk size
     10 / 20 with buffer length 4 / 5) on the same pi0.5-sized expert."""
     expert = dict(dtype=DTYPE_BF16, n_layers=18, width=1024, n_q_heads=8, head_dim=256,
                   mlp_dim=4096, action_dim=32, chunk_tokens=50)
