@@ -225,6 +225,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=20.0,
                     help="seconds of oracle work for the CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-isolated", action="store_true",
+                    help="skip the isolated-decode comparison (K passes over one chunk)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -406,6 +408,35 @@ def main():
                  "peaks": f"{peak_src}: {peaks['bf16_tflops']} TFLOP/s bf16 burst, "
                           f"{peaks['hbm_gbs']} GB/s"}
 
+    # The decode FlashVLA replaces (§1, App. A.3): pi0.5-style isolated denoising of
+    # one chunk, K passes of the same expert over [prefix ; one chunk] per emitted
+    # chunk.  Timed with the same graph replay on a K = 1 buffer of this expert.
+    isolated = None
+    if rank == 0 and wl.dtype == "bf16" and not args.no_isolated:
+        wl1 = WL.Workload(**dict(wl.__dict__, name=wl.name + "_isolated", n_chunks=1))
+        dec1 = Decoder(wl1, WL.flat_weights(wl1, w), pre)
+        b1 = torch.from_numpy(WL.make_buffer(wl1)).to(dev)
+        o1 = torch.empty((B, wl.chunk_tokens, wl.action_dim), device=dev)
+        tau1 = np.full((B, 1), 1.0 / wl.n_chunks, dtype=np.float32)
+        n1 = max(50, args.steps // 4)
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                fva.fva_step(dec1.handle, b1, tau1, o1, B, stream)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(n1):
+                fva.fva_step(dec1.handle, b1, tau1, o1, B, stream)
+            e1.record(stream)
+        torch.cuda.synchronize()
+        us1 = 1e3 * e0.elapsed_time(e1) / n1
+        dec1.close()
+        isolated = {"passes_per_chunk": wl.n_chunks, "us_per_pass": us1,
+                    "us_per_chunk": wl.n_chunks * us1, "streaming_us_per_chunk": us_per_step,
+                    "speedup": wl.n_chunks * us1 / us_per_step,
+                    "note": "K passes of the same expert over [prefix ; one chunk] per emitted "
+                            "chunk (pi0.5-style decode), against one streaming step"}
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         n_cpu, dt_cpu, cores = time_oracle(wl, w, pre, buf, tau, budget_s=args.cpu_budget,
@@ -426,9 +457,11 @@ def main():
                 "roofline": roof, "step_roofline": step_roof, "kernel_shares": shares,
                 "kernel_rooflines": kernel_rooflines,
                 "profile_note": "per-kernel times: CUDA events between the kernels of a "
-                                "captured profiling graph (event nodes serialise the "
-                                "kernels, so they include launch gaps the timed step "
-                                "hides)",
+                                "captured profiling graph; the event nodes serialise the "
+                                "kernels and cost about the same per launch, so "
+                                "(profiled step - timed step) / launches is taken off every "
+                                "launch (roofline.event_node_overhead_us)",
+                "isolated_decode": isolated,
                 "cpu_baseline": cpu}
         print(json.dumps(line))
     if dist is not None:

@@ -139,3 +139,31 @@ def test_block_diagonal_mask(dtype):
         assert_close(res["vel"], vel_ref, rel_l2=VEL_REL_L2[dtype], what="velocity")
     finally:
         case.close()
+
+
+def test_multi_buffer_forward():
+    """The packed multi-buffer forward (§3.3, App. A.4): the N cold-start
+    configurations of one observation, [pad x (N-j), j real chunks] for j = 1..N,
+    sharing one prefix and isolated from each other, in one launch as a batch of
+    N requests.  Each configuration matches the oracle, and equals running it
+    alone bit for bit (no cross-buffer interaction)."""
+    K = 3
+    base = _workload("bf16", n_chunks=K)
+    wl = WL.Workload(**dict(base.__dict__, batch=K, prefix_lens=[base.prefix_lens[0]] * K))
+    case = Case(wl)
+    try:
+        buf = np.repeat(case.buf[:1], K, axis=0)              # the same future chunks...
+        pre = [case.prefix[0]] * K                            # ...and the same observation
+        for r in range(K):
+            case.dec.set_prefix(r, pre[r][0], pre[r][1])
+        case.prefix = pre
+        n_valid = list(range(1, K + 1))
+        fresh = WL.make_fresh_noise(wl, 1)[0]
+        res = case.run(buf=buf, fresh=fresh, n_valid=n_valid)
+        check_real(res, case.oracle_step(buf=buf, fresh=fresh, n_valid=n_valid), n_valid, K, "bf16")
+        for r in range(K):
+            alone = case.run(buf=buf[r:r + 1], fresh=fresh[r:r + 1], n_valid=[n_valid[r]], batch=1)
+            c0 = K - n_valid[r]
+            np.testing.assert_array_equal(res["vel"][r, c0:], alone["vel"][0, c0:])
+    finally:
+        case.close()
