@@ -162,6 +162,7 @@ struct fva_handle {
   float2* att_part_ml = nullptr;
   int* err_dev = nullptr;
   CUtensorMap m_temb, m_t1, m_cond, m_y, m_attn, m_mlp, m_q, m_k, m_v;
+  CUtensorMap m_cond16;  // cond with 16-row boxes (streaming FiLM GEMM)
   // per-step parameters: [tau BKmax | dt BKmax | step u64]
   float* params_dev = nullptr;
   float* params_host = nullptr;  // pinned ring [FVA_PARAM_RING][params_floats]
@@ -485,6 +486,7 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
     if ((st = make_map(&h->m_temb, h->temb, BK, h->W, 128)) ||
         (st = make_map(&h->m_t1, h->t1, BK, h->W, 128)) ||
         (st = make_map(&h->m_cond, h->cond, BK, h->W, 128)) ||
+        (st = make_map(&h->m_cond16, h->cond, BK, h->W, 16)) ||
         (st = make_map(&h->m_y, h->y, M, h->W, 128)) ||
         (st = make_map(&h->m_attn, h->attn, M, h->Dq, 128)) ||
         (st = make_map(&h->m_mlp, h->mlp, M, h->F, 128)) ||
@@ -879,7 +881,10 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     ep.bias = h->b_mod;
     ep.ldo = h->N_mod;
     mark(FVA_K_FILM, -1);
-    CUDA_TRY(launch_tc_gemm(kBnFilm, GEMM_BIAS_F32, &h->m_cond, &h->m_wmod, ep, BK, h->N_mod, W, 1, s));
+    CUDA_TRY(BK <= 16 ? launch_tc_gemm_stream(&h->m_cond16, &h->m_wmod, ep, BK, h->N_mod, W,
+                                              h->n_sms, s)
+                       : launch_tc_gemm(kBnFilm, GEMM_BIAS_F32, &h->m_cond, &h->m_wmod, ep, BK,
+                                        h->N_mod, W, 1, s));
   } else {
     launch_f32_gemm((float*)h->temb, W, (float*)h->w_t1, h->c32, W, BK, W, W, s);
     launch_f32_bias_act(h->c32, h->b_t1, (float*)h->t1, BK, W, true, s);

@@ -141,6 +141,156 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ---------------------------------------------------------------------------
+// Persistent variant for weight streaming (the FiLM projection: M = B*K rows,
+// hundreds of column tiles).  One CTA per SM walks column tiles
+// blockIdx.x, blockIdx.x + gridDim.x, ...; the producer streams every tile's
+// k-blocks through one ring without draining between tiles, and the MMA
+// alternates between two TMEM accumulators so a tile's epilogue overlaps the next
+// tile's MMAs.  M <= 128 (one row tile).
+// ---------------------------------------------------------------------------
+// The condition has at most kStreamRows rows, and each stage holds only those rows
+// of A.  The M = 128 MMA reads 112 more rows past them (the stage's weights):
+// those accumulator rows are garbage and never stored, and the small A region
+// leaves room for a 6-deep weight ring.
+constexpr int kStreamRows = 16;
+
+template <int BN>
+struct GemmStreamCfg {
+  static constexpr int kABytes = kStreamRows * kBK * 2;  // 2 KB, 1024-byte aligned
+  static constexpr int kATx = kABytes;
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = 6;
+  // ring + barriers (256 B) + four 32 x 144 B epilogue stages
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256 + 4 * 32 * 144;
+};
+
+template <int BN, int MODE>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_gemm_stream_kernel(const __grid_constant__ CUtensorMap tmA,
+                          const __grid_constant__ CUtensorMap tmB, const GemmEpi ep, int M,
+                          int n_tiles, int nkb) {
+  using C = GemmStreamCfg<BN>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint64_t* full = (uint64_t*)(smem + C::kStages * C::kStageBytes);
+  uint64_t* empty = full + C::kStages;
+  uint64_t* acc_full = empty + C::kStages;  // [2]
+  uint64_t* acc_empty = acc_full + 2;       // [2]
+  uint64_t* drain = acc_empty + 2;
+  uint32_t* tmem_slot = (uint32_t*)(drain + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 4);  // one arrival per epilogue warp
+    }
+    mbar_init(drain, 1);
+    fence_barrier_init();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 2 * BN);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer: weights of the first stages before the wait
+    // the first tile's first stages: weights before waiting for the predecessor,
+    // which writes A (the condition rows)
+    const int pre = (int)blockIdx.x < n_tiles ? min(nkb, C::kStages) : 0;
+    for (int i = 0; i < pre; ++i) {
+      mbar_arrive_expect_tx(&full[i], C::kATx + C::kBBytes);
+      tma_load_2d(smem + i * C::kStageBytes + C::kABytes, &tmB, i * kBK, blockIdx.x * BN, &full[i]);
+    }
+    pdl_wait();
+    for (int i = 0; i < pre; ++i) tma_load_2d(smem + i * C::kStageBytes, &tmA, i * kBK, 0, &full[i]);
+    uint32_t it = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x) {
+      const int n0 = t * BN;
+      for (int i = 0; i < nkb; ++i, ++it) {
+        if (it < (uint32_t)pre) continue;  // issued above
+        const int s = it % C::kStages;
+        if (!mbar_wait(&empty[s], ((it / C::kStages) & 1u) ^ 1u, ep.err, KERR_WAIT_MMA)) {
+          ok = false;
+          break;
+        }
+        uint8_t* sa = smem + s * C::kStageBytes;
+        mbar_arrive_expect_tx(&full[s], C::kATx + C::kBBytes);
+        tma_load_2d(sa + C::kABytes, &tmB, i * kBK, n0, &full[s]);
+        tma_load_2d(sa, &tmA, i * kBK, 0, &full[s]);
+      }
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer
+    constexpr uint32_t idesc = umma_idesc_bf16(kBM, BN, false);
+    uint32_t it = 0, acc = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x, ++acc) {
+      const uint32_t buf = acc & 1u;
+      if (!mbar_wait(&acc_empty[buf], ((acc >> 1) & 1u) ^ 1u, ep.err, KERR_WAIT_SYNC)) break;
+      tc_fence_after();
+      const uint32_t d = tmem + buf * BN;
+      for (int i = 0; i < nkb; ++i, ++it) {
+        const int s = it % C::kStages;
+        if (!mbar_wait(&full[s], (it / C::kStages) & 1u, ep.err, KERR_WAIT_TMA)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t sa = smem_u32(smem + s * C::kStageBytes);
+        const uint32_t sb = sa + C::kABytes;
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk) {
+          const uint64_t ad = umma_desc_sw128(sa + kk * 32, 16, 1024);
+          const uint64_t bd = umma_desc_sw128(sb + kk * 32, 16, 1024);
+          umma_bf16(d, ad, bd, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+        }
+        umma_commit(&empty[s]);
+      }
+      if (ok) umma_commit(&acc_full[buf]);
+    }
+    // every MMA of this thread completes before TMEM is released
+    umma_commit(drain);
+    mbar_wait(drain, 0, nullptr, 0);
+  } else if (warp >= 2) {
+    // ---------------- epilogue: one output row per thread
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    uint8_t* stage = smem + C::kStages * C::kStageBytes + 256 + (warp - 2) * (32 * 144);
+    uint32_t acc = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++acc) {
+      const uint32_t buf = acc & 1u;
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (acc >> 1) & 1u, ep.err,
+                                                     KERR_WAIT_MMA));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t trow = tmem + buf * BN + ((uint32_t)(quarter * 32) << 16);
+      gemm_epilogue<BN, MODE>(ep, trow, row, M, t * BN, 0, stage, lane);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[buf]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 2 * BN);
+  }
+}
+
 template <int BN, int MODE>
 cudaError_t set_attr() {
   return cudaFuncSetAttribute(tc_gemm_kernel<BN, MODE>,
@@ -162,6 +312,10 @@ cudaError_t launch(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep
 
 cudaError_t tc_gemm_init() {
   cudaError_t e;
+  if ((e = cudaFuncSetAttribute(tc_gemm_stream_kernel<kBnFilm, GEMM_BIAS_F32>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                GemmStreamCfg<kBnFilm>::kSmemBytes)) != cudaSuccess)
+    return e;
   if ((e = set_attr<kBnTime, GEMM_BIAS_SILU_BF16>()) != cudaSuccess) return e;
   if ((e = set_attr<kBnFilm, GEMM_BIAS_F32>()) != cudaSuccess) return e;
   if ((e = set_attr<kBnQKV, GEMM_QKV_ROPE>()) != cudaSuccess) return e;
@@ -185,6 +339,20 @@ cudaError_t launch_tc_gemm(int bn, int mode, const CUtensorMap* a, const CUtenso
   if (bn == kBnGU && mode == GEMM_GEGLU)
     return launch<kBnGU, GEMM_GEGLU>(a, b, ep, M, N, K, splits, s);
   return cudaErrorInvalidValue;
+}
+
+}  // namespace fva
+
+namespace fva {
+
+cudaError_t launch_tc_gemm_stream(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep,
+                                  int M, int N, int K, int grid, cudaStream_t s) {
+  if (M <= 0 || N <= 0) return cudaSuccess;
+  if (M > kStreamRows || N % kBnFilm != 0 || K % kBK != 0) return cudaErrorInvalidValue;
+  const int n_tiles = N / kBnFilm;
+  return launch_pdl(tc_gemm_stream_kernel<kBnFilm, GEMM_BIAS_F32>, dim3(std::min(grid, n_tiles)),
+                    dim3(kThreads), GemmStreamCfg<kBnFilm>::kSmemBytes, s, *a, *b, ep, M, n_tiles,
+                    K / kBK);
 }
 
 }  // namespace fva
