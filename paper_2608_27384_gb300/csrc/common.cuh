@@ -134,38 +134,6 @@ __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* m
       : "memory");
 }
 
-// Ask the memory system to bring [addr, addr + bytes) into L2 (fire and forget).
-// addr and bytes must be multiples of 16.
-__device__ __forceinline__ void prefetch_l2_bulk(const void* addr, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(addr), "r"(bytes) : "memory");
-}
-
-// Up to three byte ranges to prefetch into L2, split into 64 KiB pieces that the
-// CTAs of a grid issue round-robin (thread 0 of each CTA).
-struct L2Prefetch {
-  const void* ptr[3];
-  unsigned long long bytes[3];
-};
-
-__device__ __forceinline__ void issue_l2_prefetch(const L2Prefetch& pf) {
-  if (threadIdx.x != 0) return;
-  constexpr unsigned long long kPiece = 65536;
-  unsigned long long base = 0;
-  for (int r = 0; r < 3; ++r) {
-    const unsigned long long n = pf.bytes[r];
-    if (!pf.ptr[r] || n == 0) continue;
-    const unsigned long long pieces = (n + kPiece - 1) / kPiece;
-    // piece i of this range has global index base + i; CTA b takes indices = b mod grid
-    unsigned long long first = (blockIdx.x + gridDim.x - base % gridDim.x) % gridDim.x;
-    for (unsigned long long i = first; i < pieces; i += gridDim.x) {
-      const unsigned long long off = i * kPiece;
-      const unsigned long long len = (n - off < kPiece) ? (n - off) : kPiece;
-      prefetch_l2_bulk((const uint8_t*)pf.ptr[r] + off, (uint32_t)(len & ~15ull));
-    }
-    base += pieces;
-  }
-}
-
 // ----------------------------------------------------------------------------
 // tcgen05: tensor memory, UMMA descriptors, MMA, commit, loads
 // ----------------------------------------------------------------------------

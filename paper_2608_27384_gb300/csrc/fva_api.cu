@@ -897,34 +897,8 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
 
   // ---- action in-projection + layer 0 norm 1
   mark(FVA_K_EMBED_NORM, -1);
-  {
-    L2Prefetch pf0{};
-    const LayerW& lw = h->layers[0];
-    pf0.ptr[0] = lw.w_qkv;
-    pf0.bytes[0] = (unsigned long long)((const uint8_t*)lw.w_d - (const uint8_t*)lw.w_qkv) +
-                   (unsigned long long)W * F * a;
-    pf0.ptr[1] = h->kc;
-    pf0.bytes[1] = (size_t)B * h->S_cap * h->dh * a;
-    pf0.ptr[2] = h->vc;
-    pf0.bytes[2] = pf0.bytes[1];
-    launch_embed_norm(d, buffer, h->w_in_t, h->b_in, h->mod, h->h, h->y, bf, &pf0, s);
-  }
+  launch_embed_norm(d, buffer, h->w_in_t, h->b_in, h->mod, h->h, h->y, bf, s);
 
-  // L2 prefetch of layer l's weights and prefix/action K/V, issued by the norm
-  // kernel that precedes the layer (it runs while the previous GEMM drains).
-  const size_t kv_bytes_layer = (size_t)B * h->S_cap * h->dh * a;
-  auto layer_prefetch = [&](int l) {
-    L2Prefetch pf{};
-    const LayerW& lw = h->layers[l];
-    pf.ptr[0] = lw.w_qkv;
-    pf.bytes[0] = (unsigned long long)((const uint8_t*)lw.w_d - (const uint8_t*)lw.w_qkv) +
-                  (unsigned long long)W * F * a;
-    pf.ptr[1] = (const uint8_t*)h->kc + (size_t)l * kv_layer * a;
-    pf.bytes[1] = kv_bytes_layer;
-    pf.ptr[2] = (const uint8_t*)h->vc + (size_t)l * kv_layer * a;
-    pf.bytes[2] = kv_bytes_layer;
-    return pf;
-  };
   const int m_tiles = (M + 127) / 128;
   const int sp_o = bf ? choose_splits(m_tiles * (W / kBnResid), Dq / 64) : 1;
   const int sp_d = bf ? choose_splits(m_tiles * (W / kBnResid), F / 64) : 1;
@@ -1062,7 +1036,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     }
     mark(FVA_K_RESID_NORM, l);
     launch_resid_norm(d, h->h, h->part, sp_o, pstride, h->mod, mod_off(l, 2, W), mod_off(l, 3, W),
-                      mod_off(l, 4, W), h->y, bf, nullptr, s);
+                      mod_off(l, 4, W), h->y, bf, s);
     if (trace) {
       CUDA_TRY(copy_h(o_hmid));
       launch_to_f32(h->y, bf, tr_at(o_y2), (long long)MW, s);
@@ -1088,9 +1062,8 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     if (trace) launch_to_f32(h->mlp, bf, tr_at(o_mlp), (long long)M * F, s);
     if (l + 1 < L) {
       mark(FVA_K_RESID_NORM, l);
-      const L2Prefetch pf = layer_prefetch(l + 1);
       launch_resid_norm(d, h->h, h->part, sp_d, pstride, h->mod, mod_off(l, 5, W),
-                        mod_off(l + 1, 0, W), mod_off(l + 1, 1, W), h->y, bf, &pf, s);
+                        mod_off(l + 1, 0, W), mod_off(l + 1, 1, W), h->y, bf, s);
       if (trace) CUDA_TRY(copy_h(o_hout));
     }
   }

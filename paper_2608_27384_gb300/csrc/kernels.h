@@ -44,19 +44,14 @@ void set_last_error(const char* msg);
 void launch_temb(const float* tau, const float2* freq, int rows, int W, void* out,
                  bool act_bf16, cudaStream_t s);
 
-struct L2Prefetch;
-
-// pf (nullable): byte ranges the kernel's CTAs prefetch into L2 before waiting
-// on their predecessor (the next layer's weights and prefix K/V).
 void launch_embed_norm(const StepDims& d, const float* buffer, const float* w_in_t,
                        const float* b_in, const float* mod, float* h, void* y, bool act_bf16,
-                       const L2Prefetch* pf, cudaStream_t s);
+                       cudaStream_t s);
 
 // h += gate * sum_z part[z];  y = rmsnorm(h) * (1 + scale) + shift.
 void launch_resid_norm(const StepDims& d, float* h, const float* part, int n_parts,
                        long long part_stride, const float* mod, int gate_off, int scale_off,
-                       int shift_off, void* y, bool act_bf16, const L2Prefetch* pf,
-                       cudaStream_t s);
+                       int shift_off, void* y, bool act_bf16, cudaStream_t s);
 
 // Final residual + final FiLM RMSNorm (fp32 y_F into yF [B*K*H, W]), then
 // out-projection, Euler update, emit, roll and tail (two launches).  w_out_t is

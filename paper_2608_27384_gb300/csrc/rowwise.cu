@@ -113,14 +113,12 @@ template <typename Act>
 __global__ void embed_norm_kernel(StepDims d, const float* __restrict__ buffer,
                                   const float* __restrict__ w_in_t,
                                   const float* __restrict__ b_in, const float* __restrict__ mod,
-                                  float* __restrict__ h, Act* __restrict__ y,
-                                  const L2Prefetch pf) {
+                                  float* __restrict__ h, Act* __restrict__ y) {
   __shared__ float xs[128];
   __shared__ float red[32];
   const int m = blockIdx.x;
   const int r = m / d.T, t = m % d.T, c = t / d.H;
   pdl_trigger();
-  issue_l2_prefetch(pf);
   pdl_wait();
   const float* x = buffer + (size_t)m * d.A;  // buffer [B, K, H, A] = rows of A
   for (int a = threadIdx.x; a < d.A; a += blockDim.x) xs[a] = x[a];
@@ -148,16 +146,15 @@ __global__ void embed_norm_kernel(StepDims d, const float* __restrict__ buffer,
 
 void launch_embed_norm(const StepDims& d, const float* buffer, const float* w_in_t,
                        const float* b_in, const float* mod, float* h, void* y, bool act_bf16,
-                       const L2Prefetch* pf, cudaStream_t s) {
+                       cudaStream_t s) {
   const int rows = d.B * d.T;
   if (rows <= 0) return;
-  const L2Prefetch none = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
   if (act_bf16)
     launch_pdl(embed_norm_kernel<bf16>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, buffer,
-               w_in_t, b_in, mod, h, (bf16*)y, pf ? *pf : none);
+               w_in_t, b_in, mod, h, (bf16*)y);
   else
     launch_pdl(embed_norm_kernel<float>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, buffer,
-               w_in_t, b_in, mod, h, (float*)y, pf ? *pf : none);
+               w_in_t, b_in, mod, h, (float*)y);
 }
 
 // ----------------------------------------------------------------------------
@@ -169,12 +166,11 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
                                   const float* __restrict__ part, int n_parts,
                                   long long part_stride, const float* __restrict__ mod,
                                   int gate_off, int scale_off, int shift_off,
-                                  Act* __restrict__ y, const L2Prefetch pf) {
+                                  Act* __restrict__ y) {
   __shared__ float red[32];
   const int m = blockIdx.x;
   const int r = m / d.T, c = (m % d.T) / d.H;
   pdl_trigger();
-  issue_l2_prefetch(pf);
   pdl_wait();
   const float* mrow = mod + (size_t)(r * d.K + c) * d.N_mod;
   float* hrow = h + (size_t)m * d.W;
@@ -236,19 +232,15 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
 
 void launch_resid_norm(const StepDims& d, float* h, const float* part, int n_parts,
                        long long part_stride, const float* mod, int gate_off, int scale_off,
-                       int shift_off, void* y, bool act_bf16, const L2Prefetch* pf,
-                       cudaStream_t s) {
+                       int shift_off, void* y, bool act_bf16, cudaStream_t s) {
   const int rows = d.B * d.T;
   if (rows <= 0) return;
-  const L2Prefetch none = {{nullptr, nullptr, nullptr}, {0, 0, 0}};
   if (act_bf16)
     launch_pdl(resid_norm_kernel<bf16>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h, part,
-               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (bf16*)y,
-               pf ? *pf : none);
+               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (bf16*)y);
   else
     launch_pdl(resid_norm_kernel<float>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h, part,
-               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (float*)y,
-               pf ? *pf : none);
+               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (float*)y);
 }
 
 // ----------------------------------------------------------------------------
@@ -430,7 +422,7 @@ cudaError_t final_init(const StepDims& d) {
 void launch_final_norm(const StepDims& d, float* h, const float* part, int n_parts,
                        long long part_stride, const float* mod, float* yF, cudaStream_t s) {
   launch_resid_norm(d, h, part, n_parts, part_stride, mod, mod_off(d.L - 1, 5, d.W),
-                    modf_off(d.L, 0, d.W), modf_off(d.L, 1, d.W), yF, false, nullptr, s);
+                    modf_off(d.L, 0, d.W), modf_off(d.L, 1, d.W), yF, false, s);
 }
 
 void launch_velocity_euler(const StepDims& d, const float* yF, const float* w_out_t,
