@@ -123,6 +123,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------- epilogue: warp w reads TMEM lanes 32*(w%4) .. +31
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;
+    if constexpr (MODE == GEMM_QKV_ROPE) gemm_epilogue_prefetch_rope<BN>(ep, m0 + row, M, n0);
     const bool good = __all_sync(0xffffffffu, mbar_wait(acc_full, 0, ep.err, KERR_WAIT_MMA));
     tc_fence_after();
     if (good && nkb > 0) {
