@@ -214,6 +214,47 @@ def time_oracle(wl, w, pre, buf, tau, budget_s: float, max_steps: int):
 
 # ---------------------------------------------------------------------------
 
+class Replicas:
+    """The multi-GPU form of the step: independent replicas, one per rank (requests
+    shard by rank; no collective on the data path).  The only cross-rank traffic
+    is the harness's barrier around the timed region and the max over ranks of
+    its duration.  backend "nccl" on GPUs; "gloo" serves the CPU tests."""
+
+    def __init__(self, world: int, backend: str, device):
+        import torch
+        self.torch = torch
+        self.device = device
+        self.dist = None
+        if world > 1:
+            import torch.distributed as dist
+            if backend == "nccl":
+                dist.init_process_group(backend, device_id=device)
+            else:
+                dist.init_process_group(backend)
+            self.dist = dist
+
+    def _sync(self):
+        if self.device.type == "cuda":
+            self.torch.cuda.synchronize(self.device)
+
+    def barrier(self):
+        self._sync()
+        if self.dist is not None:
+            self.dist.barrier()
+        self._sync()
+
+    def max(self, x: float) -> float:
+        if self.dist is None:
+            return x
+        t = self.torch.tensor([x], device=self.device, dtype=self.torch.float64)
+        self.dist.all_reduce(t, op=self.dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.dist is not None:
+            self.dist.destroy_process_group()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -268,14 +309,9 @@ def main():
     import paper_2608_27384_gb300 as fva
     from paper_2608_27384_gb300.harness import Decoder
 
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        torch.cuda.set_device(local_rank)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
-    else:
-        torch.cuda.set_device(0)
+    torch.cuda.set_device(local_rank if world > 1 else 0)
     dev = torch.device("cuda", local_rank if world > 1 else 0)
+    replicas = Replicas(world, "nccl", dev)
 
     w = WL.make_weights(wl)
     pre = WL.make_prefix_kv(wl)
@@ -288,18 +324,8 @@ def main():
     d_buf = torch.from_numpy(buf).to(dev)
     d_out = torch.empty((B, wl.chunk_tokens, wl.action_dim), device=dev)
 
-    def barrier():
-        torch.cuda.synchronize()
-        if dist is not None:
-            dist.barrier()
-        torch.cuda.synchronize()
-
-    def max_over_ranks(x: float) -> float:
-        if dist is None:
-            return x
-        t = torch.tensor([x], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+    barrier = replicas.barrier
+    max_over_ranks = replicas.max
 
     # ---- device-resident timing: graph replay through fva_step
     with torch.cuda.stream(stream):
@@ -464,8 +490,7 @@ def main():
                 "isolated_decode": isolated,
                 "cpu_baseline": cpu}
         print(json.dumps(line))
-    if dist is not None:
-        dist.destroy_process_group()
+    replicas.close()
     return 0
 
 
