@@ -585,6 +585,9 @@ __global__ void __launch_bounds__(kThreads, 1) block_kernel(const __grid_constan
       }
     }
   }
+  // the producer and MMA lanes rejoin their warps first: a CTA barrier reached
+  // by a split warp does not wait for the rest of the CTA
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {

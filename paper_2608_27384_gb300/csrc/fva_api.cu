@@ -873,10 +873,26 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   GemmEpi ep{};
   ep.err = h->err_dev;
   if (bf) {
-    mark(FVA_K_TIME_MLP, -1);
-    launch_gemv_silu(h->temb, h->w_t1, h->b_t1, h->t1, BK, W, W, s);
-    mark(FVA_K_TIME_MLP, -1);
-    launch_gemv_silu(h->t1, h->w_t2, h->b_t2, h->cond, BK, W, W, s);
+    // a few rows: one warp per output column (GEMV); more: the tensor-core GEMM
+    // (the GEMV walks its rows 16 at a time)
+    if (BK <= 32) {
+      mark(FVA_K_TIME_MLP, -1);
+      launch_gemv_silu(h->temb, h->w_t1, h->b_t1, h->t1, BK, W, W, s);
+      mark(FVA_K_TIME_MLP, -1);
+      launch_gemv_silu(h->t1, h->w_t2, h->b_t2, h->cond, BK, W, W, s);
+    } else {
+      GemmEpi et{};
+      et.err = h->err_dev;
+      et.out = h->t1;
+      et.bias = h->b_t1;
+      et.ldo = W;
+      mark(FVA_K_TIME_MLP, -1);
+      CUDA_TRY(launch_tc_gemm(kBnTime, GEMM_BIAS_SILU_BF16, &h->m_temb, &h->m_wt1, et, BK, W, W, 1, s));
+      et.out = h->cond;
+      et.bias = h->b_t2;
+      mark(FVA_K_TIME_MLP, -1);
+      CUDA_TRY(launch_tc_gemm(kBnTime, GEMM_BIAS_SILU_BF16, &h->m_t1, &h->m_wt2, et, BK, W, W, 1, s));
+    }
     ep.out = h->mod;
     ep.bias = h->b_mod;
     ep.ldo = h->N_mod;
@@ -897,7 +913,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
 
   // ---- action in-projection + layer 0 norm 1
   mark(FVA_K_EMBED_NORM, -1);
-  launch_embed_norm(d, buffer, h->w_in_t, h->b_in, h->mod, h->h, h->y, bf, s);
+  launch_embed_norm(d, buffer, h->w_in_t, h->b_in, h->mod, h->h, h->y, bf, h->n_sms, s);
 
   const int m_tiles = (M + 127) / 128;
   const int sp_o = bf ? choose_splits(m_tiles * (W / kBnResid), Dq / 64) : 1;

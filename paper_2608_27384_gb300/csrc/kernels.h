@@ -46,7 +46,7 @@ void launch_temb(const float* tau, const float2* freq, int rows, int W, void* ou
 
 void launch_embed_norm(const StepDims& d, const float* buffer, const float* w_in_t,
                        const float* b_in, const float* mod, float* h, void* y, bool act_bf16,
-                       cudaStream_t s);
+                       int n_sms, cudaStream_t s);
 
 // h += gate * sum_z part[z];  y = rmsnorm(h) * (1 + scale) + shift.
 void launch_resid_norm(const StepDims& d, float* h, const float* part, int n_parts,

@@ -107,54 +107,108 @@ inline int row_threads(int W) {
 
 // ----------------------------------------------------------------------------
 // action in-projection h = x W_in^T + b_in, then layer 0's FiLM RMSNorm.
-// One CTA per token row; w_in_t is W_in transposed, [A, W] fp32.
+// R token rows per CTA, so each CTA reads w_in_t (W_in transposed, [A, W] fp32)
+// once for all of them; each thread owns 4 columns of every row.
 // ----------------------------------------------------------------------------
-template <typename Act>
-__global__ void embed_norm_kernel(StepDims d, const float* __restrict__ buffer,
+template <typename Act, int R>
+__global__ void embed_norm_kernel(StepDims d, int rows, const float* __restrict__ buffer,
                                   const float* __restrict__ w_in_t,
                                   const float* __restrict__ b_in, const float* __restrict__ mod,
                                   float* __restrict__ h, Act* __restrict__ y) {
-  __shared__ float xs[128];
+  __shared__ float xs[R][128];
   __shared__ float red[32];
-  const int m = blockIdx.x;
-  const int r = m / d.T, t = m % d.T, c = t / d.H;
+  const int m0 = blockIdx.x * R;
+  const int nr = min(R, rows - m0);
   pdl_trigger();
   pdl_wait();
-  const float* x = buffer + (size_t)m * d.A;  // buffer [B, K, H, A] = rows of A
-  for (int a = threadIdx.x; a < d.A; a += blockDim.x) xs[a] = x[a];
-  __syncthreads();
-  float* hrow = h + (size_t)m * d.W;
-  float ss = 0.f;
-  for (int col = threadIdx.x * 4; col < d.W; col += blockDim.x * 4) {
-    float4 acc = *reinterpret_cast<const float4*>(b_in + col);
-    for (int a = 0; a < d.A; ++a) {
-      const float xa = xs[a];
-      const float4 w = *reinterpret_cast<const float4*>(w_in_t + (size_t)a * d.W + col);
-      acc.x = fmaf(xa, w.x, acc.x);
-      acc.y = fmaf(xa, w.y, acc.y);
-      acc.z = fmaf(xa, w.z, acc.z);
-      acc.w = fmaf(xa, w.w, acc.w);
-    }
-    *reinterpret_cast<float4*>(hrow + col) = acc;
-    ss += acc.x * acc.x + acc.y * acc.y + acc.z * acc.z + acc.w * acc.w;
+  // buffer [B, K, H, A] = rows of A, token rows m0 .. m0 + nr - 1 contiguous
+  for (int i = threadIdx.x; i < R * d.A; i += blockDim.x) {
+    const int r = i / d.A, a = i % d.A;
+    xs[r][a] = r < nr ? buffer[(size_t)(m0 + r) * d.A + a] : 0.f;
   }
-  ss = block_sum(ss, red);
-  const float* mrow = mod + (size_t)(r * d.K + c) * d.N_mod;
-  modulated_norm_row<Act>(hrow, ss, d.W, d.eps, mrow + mod_off(0, 0, d.W),
-                          mrow + mod_off(0, 1, d.W), y + (size_t)m * d.W);
+  __syncthreads();
+  float ss[R];
+#pragma unroll
+  for (int r = 0; r < R; ++r) ss[r] = 0.f;
+  for (int col = threadIdx.x * 4; col < d.W; col += blockDim.x * 4) {
+    float4 acc[R];
+    const float4 bias = *reinterpret_cast<const float4*>(b_in + col);
+#pragma unroll
+    for (int r = 0; r < R; ++r) acc[r] = bias;
+    // 16 weight loads in flight per thread before the FMAs (one CTA per SM has to
+    // cover the L2 latency on its own)
+    for (int a0 = 0; a0 < d.A; a0 += 16) {
+      float4 w[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j)
+        if (a0 + j < d.A) w[j] = *reinterpret_cast<const float4*>(w_in_t + (size_t)(a0 + j) * d.W + col);
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        if (a0 + j >= d.A) break;
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+          const float xa = xs[r][a0 + j];
+          acc[r].x = fmaf(xa, w[j].x, acc[r].x);
+          acc[r].y = fmaf(xa, w[j].y, acc[r].y);
+          acc[r].z = fmaf(xa, w[j].z, acc[r].z);
+          acc[r].w = fmaf(xa, w[j].w, acc[r].w);
+        }
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+      if (r < nr) {
+        *reinterpret_cast<float4*>(h + (size_t)(m0 + r) * d.W + col) = acc[r];
+        ss[r] += acc[r].x * acc[r].x + acc[r].y * acc[r].y + acc[r].z * acc[r].z +
+                 acc[r].w * acc[r].w;
+      }
+  }
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    if (r >= nr) break;  // uniform over the CTA
+    const int m = m0 + r;
+    const int rq = m / d.T, c = (m % d.T) / d.H;
+    const float tot = block_sum(ss[r], red);
+    const float* mrow = mod + (size_t)(rq * d.K + c) * d.N_mod;
+    modulated_norm_row<Act>(h + (size_t)m * d.W, tot, d.W, d.eps, mrow + mod_off(0, 0, d.W),
+                            mrow + mod_off(0, 1, d.W), y + (size_t)m * d.W);
+  }
+}
+
+template <typename Act, int R>
+static void launch_embed_norm_r(const StepDims& d, int rows, const float* buffer,
+                                const float* w_in_t, const float* b_in, const float* mod,
+                                float* h, Act* y, cudaStream_t s) {
+  launch_pdl(embed_norm_kernel<Act, R>, dim3((rows + R - 1) / R), dim3(row_threads(d.W)), 0, s,
+             d, rows, buffer, w_in_t, b_in, mod, h, y);
+}
+
+template <typename Act>
+static void launch_embed_norm_t(const StepDims& d, int rows, int n_sms, const float* buffer,
+                                const float* w_in_t, const float* b_in, const float* mod,
+                                float* h, Act* y, cudaStream_t s) {
+  // rows per CTA: about one CTA per SM, so w_in_t is read about once per SM
+  const int per_sm = (rows + n_sms - 1) / n_sms;
+  if (per_sm >= 8)
+    launch_embed_norm_r<Act, 8>(d, rows, buffer, w_in_t, b_in, mod, h, y, s);
+  else if (per_sm >= 4)
+    launch_embed_norm_r<Act, 4>(d, rows, buffer, w_in_t, b_in, mod, h, y, s);
+  else if (per_sm >= 2)
+    launch_embed_norm_r<Act, 2>(d, rows, buffer, w_in_t, b_in, mod, h, y, s);
+  else
+    launch_embed_norm_r<Act, 1>(d, rows, buffer, w_in_t, b_in, mod, h, y, s);
 }
 
 void launch_embed_norm(const StepDims& d, const float* buffer, const float* w_in_t,
                        const float* b_in, const float* mod, float* h, void* y, bool act_bf16,
-                       cudaStream_t s) {
+                       int n_sms, cudaStream_t s) {
   const int rows = d.B * d.T;
   if (rows <= 0) return;
+  if (n_sms < 1) n_sms = 1;
   if (act_bf16)
-    launch_pdl(embed_norm_kernel<bf16>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, buffer,
-               w_in_t, b_in, mod, h, (bf16*)y);
+    launch_embed_norm_t<bf16>(d, rows, n_sms, buffer, w_in_t, b_in, mod, h, (bf16*)y, s);
   else
-    launch_pdl(embed_norm_kernel<float>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, buffer,
-               w_in_t, b_in, mod, h, (float*)y);
+    launch_embed_norm_t<float>(d, rows, n_sms, buffer, w_in_t, b_in, mod, h, (float*)y, s);
 }
 
 // ----------------------------------------------------------------------------

@@ -10,19 +10,19 @@
 // tile in shared memory serves every head.  The key range of a tile is cut into
 // splits of 256 keys (4 blocks of 64); key blocks past the tile's largest limit
 // are never loaded.  One CTA handles one (tile, split):
-//   warp 0      TMA: the Q tile (64 KB) and all K blocks at once, then the V
-//               blocks as K slots free up (4-slot ring of 32 KB);
+//   warp 0      TMA: the Q tile (64 KB) and the split's K blocks, then, once
+//               the S MMAs have read K, the V blocks into the same space;
 //   warp 1      TMEM (512 columns: S in 0..255, O in 256..511); one lane issues
-//               S = Q K^T per key block (M=128, N=64, K=16 steps over dh), and,
+//               S = Q K^T as one MMA per 16 head dims with N = all the split's
+//               keys (each Q and K byte is read from shared memory once), and,
 //               after the softmax, O = P V (M=128, N=256, MN-major V);
 //   warps 2..17 softmax + epilogue, four threads per query row (one per
-//               64-key block / 64 head-dim columns).  As soon as its block of S
-//               is in TMEM a thread takes the block's row max over visible keys
-//               and writes P = exp(S - block max) as bf16 over the Q tile (Q is
-//               dead once S is complete); after the four threads of a row
-//               exchange maxima it rescales its P block by exp(block max - row
-//               max) in place, so the exponentials overlap the S MMAs of later
-//               blocks.  Then O is read from TMEM.
+//               64-key block / 64 head-dim columns): block max, row max through
+//               shared memory, P = exp(S - row max) as bf16 over the Q tile (Q is
+//               dead once S is complete) with the row's sum; then O from TMEM.
+// K and V live slab-major: head-dim slab j (64 values, 128 bytes) of key k is
+// at j * 32 KB + k * 128 bytes, so the split's keys form one uniformly strided
+// operand for the S MMA and V's head-dim slabs are 32 KB apart for the P V MMA.
 // A tile with one split writes O / l as bf16.  Otherwise each split writes O / l
 // (bf16) and its (max, sum) to scratch and attn_merge_kernel combines the splits
 // of every row in split order (deterministic) and writes bf16.
@@ -39,12 +39,19 @@ constexpr int kKB = kAttnKeyBlock;                        // 64 keys per block
 constexpr int kBlocksPerSplit = kAttnKeysPerSplit / kKB;  // 4
 constexpr int kQBytes = kRows * kDH * 2;                  // 64 KB (Q, later P)
 constexpr int kKVBytes = kKB * kDH * 2;                   // 32 KB per K or V block
-constexpr int kSlots = 4;
 constexpr int kSoftmaxThreads = 512;
 constexpr int kThreads = 64 + kSoftmaxThreads;
-constexpr int kSmem = kQBytes + kSlots * kKVBytes + 1024 /*align*/ + 1024 /*bars*/ +
+constexpr int kSmem = kQBytes + kBlocksPerSplit * kKVBytes + 1024 /*align*/ + 1024 /*bars*/ +
                       8 * kRows * 4 /*row exchange*/;
 constexpr uint32_t kTmemCols = 512;
+
+// 2^x by the PTX ex2.approx.ftz.f32 instruction (relative error about 2^-22,
+// far below the bf16 rounding P gets next; results below 2^-126 flush to 0)
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 __device__ __forceinline__ void softmax_bar() {
   asm volatile("bar.sync 1, 512;" ::: "memory");
@@ -72,14 +79,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* sQP = smem;                      // 4 slabs [128 rows x 128 B]: Q, then P
-  uint8_t* sKV = smem + kQBytes;            // 4 slots x 4 slabs [64 rows x 128 B]
-  uint64_t* bars = (uint64_t*)(sKV + kSlots * kKVBytes);
+  uint8_t* sKV = smem + kQBytes;            // 4 slabs [256 keys x 128 B]: K, then V
+  uint64_t* bars = (uint64_t*)(sKV + kBlocksPerSplit * kKVBytes);
   uint64_t* q_full = bars + 0;
-  uint64_t* kv_full = bars + 1;   // [4]
-  uint64_t* kv_empty = bars + 5;  // [4]
-  uint64_t* s_full = bars + 9;    // [4]: block g of S is in TMEM
-  uint64_t* p_full = bars + 13;
-  uint64_t* o_full = bars + 14;
+  uint64_t* kv_full = bars + 1;   // [4]: key block b of K (phase 0), then of V (phase 1)
+  uint64_t* k_free = bars + 5;    // the S MMAs have read K
+  uint64_t* s_full = bars + 6;    // S is in TMEM
+  uint64_t* p_full = bars + 7;
+  uint64_t* o_full = bars + 8;
   uint32_t* tmem_slot = (uint32_t*)(bars + 15);
   float* xmax = (float*)(bars + 128);   // [4][128] per-block row max
   float* xsum = xmax + 4 * kRows;       // [4][128] per-block row sum
@@ -87,11 +94,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int s = 0; s < kSlots; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
-    }
-    for (int g = 0; g < kBlocksPerSplit; ++g) mbar_init(&s_full[g], 1);
+    for (int b = 0; b < kBlocksPerSplit; ++b) mbar_init(&kv_full[b], 1);
+    mbar_init(k_free, 1);
+    mbar_init(s_full, 1);
     mbar_init(p_full, kSoftmaxThreads);
     mbar_init(o_full, 1);
     fence_barrier_init();
@@ -118,70 +123,56 @@ __global__ void __launch_bounds__(kThreads, 1)
     // not from the predecessor grid, so they are requested before waiting for
     // it; q and the action keys/values (written by the QKV projection) after.
     // Every other thread only runs behind these loads.
-    int it = 0;
-    for (; it < nblk && (kb0 + it + 1) * kKB <= P; ++it) {  // first use of slot it
-      mbar_arrive_expect_tx(&kv_full[it], kKVBytes);
+    auto load_block = [&](const CUtensorMap* map, int b) {
+      mbar_arrive_expect_tx(&kv_full[b], kKVBytes);
       for (int j = 0; j < 4; ++j)
-        tma_load_2d(sKV + it * kKVBytes + j * (kKB * 128), &tmK, j * 64, krow0 + it * kKB,
-                    &kv_full[it]);
-    }
+        tma_load_2d(sKV + j * (kBlocksPerSplit * kKB * 128) + b * (kKB * 128), map, j * 64,
+                    krow0 + b * kKB, &kv_full[b]);
+    };
+    int b = 0;
+    for (; b < nblk && (kb0 + b + 1) * kKB <= P; ++b) load_block(&tmK, b);
     pdl_wait();
     mbar_arrive_expect_tx(q_full, kQBytes);
     for (int j = 0; j < 4; ++j) tma_load_2d(sQP + j * (kRows * 128), &tmQ, j * 64, qrow0, q_full);
-    for (; it < 2 * nblk; ++it) {
-      const int s = it % kSlots;
-      const uint32_t ph = (uint32_t)(it / kSlots) & 1u;
-      if (!mbar_wait(&kv_empty[s], ph ^ 1u, a.err, KERR_WAIT_MMA)) break;
-      const bool is_k = it < nblk;
-      const int row = krow0 + (is_k ? it : it - nblk) * kKB;
-      uint8_t* dst = sKV + s * kKVBytes;
-      mbar_arrive_expect_tx(&kv_full[s], kKVBytes);
-      for (int j = 0; j < 4; ++j)
-        tma_load_2d(dst + j * (kKB * 128), is_k ? &tmK : &tmV, j * 64, row, &kv_full[s]);
-    }
+    for (; b < nblk; ++b) load_block(&tmK, b);
+    if (mbar_wait(k_free, 0, a.err, KERR_WAIT_MMA))
+      for (b = 0; b < nblk; ++b) load_block(&tmV, b);
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer
-    constexpr uint32_t idesc_s = umma_idesc_bf16(kRows, kKB, false);
+    const uint32_t idesc_s = umma_idesc_bf16(kRows, nblk * kKB, false);
     constexpr uint32_t idesc_o = umma_idesc_bf16(kRows, kDH, true);
+    constexpr uint32_t kSlabK = kBlocksPerSplit * kKB * 128;  // 32 KB between head-dim slabs
     bool good = mbar_wait(q_full, 0, a.err, KERR_WAIT_TMA);
+    for (int b = 0; good && b < nblk; ++b) good = mbar_wait(&kv_full[b], 0, a.err, KERR_WAIT_TMA);
     tc_fence_after();
     const uint32_t qp_base = smem_u32(sQP), kv_base = smem_u32(sKV);
-    for (int it = 0; good && it < nblk; ++it) {
-      const int s = it % kSlots;
-      if (!mbar_wait(&kv_full[s], (uint32_t)(it / kSlots) & 1u, a.err, KERR_WAIT_TMA)) {
-        good = false;
-        break;
-      }
-      tc_fence_after();
-      const uint32_t kb = kv_base + s * kKVBytes;
+    if (good) {
 #pragma unroll
       for (int ks = 0; ks < kDH / 16; ++ks) {
         const uint32_t off = (ks & 3) * 32;  // 16 bf16 along K inside the 128-byte row
         const uint64_t ad = umma_desc_sw128(qp_base + (ks >> 2) * (kRows * 128) + off, 16, 1024);
-        const uint64_t bd = umma_desc_sw128(kb + (ks >> 2) * (kKB * 128) + off, 16, 1024);
-        umma_bf16(tS + it * kKB, ad, bd, idesc_s, ks > 0 ? 1u : 0u);
+        const uint64_t bd = umma_desc_sw128(kv_base + (ks >> 2) * kSlabK + off, 16, 1024);
+        umma_bf16(tS, ad, bd, idesc_s, ks > 0 ? 1u : 0u);
       }
-      umma_commit(&kv_empty[s]);
-      umma_commit(&s_full[it]);
+      umma_commit(k_free);
+      umma_commit(s_full);
     }
     if (good) good = mbar_wait(p_full, 0, a.err, KERR_WAIT_SYNC);
     tc_fence_after();
     for (int j = 0; good && j < nblk; ++j) {
-      const int it = nblk + j, s = it % kSlots;
-      if (!mbar_wait(&kv_full[s], (uint32_t)(it / kSlots) & 1u, a.err, KERR_WAIT_TMA)) {
+      if (!mbar_wait(&kv_full[j], 1, a.err, KERR_WAIT_TMA)) {
         good = false;
         break;
       }
       tc_fence_after();
-      const uint32_t vb = kv_base + s * kKVBytes;
 #pragma unroll
       for (int ks = 0; ks < kKB / 16; ++ks) {
         const uint64_t ad = umma_desc_sw128(qp_base + j * (kRows * 128) + ks * 32, 16, 1024);
-        // V block [64 keys][256 dh] as 4 slabs of 64 dh: MN-major B operand.
-        const uint64_t bd = umma_desc_sw128(vb + ks * 16 * 128, kKB * 128, 1024);
+        // V keys j*64 + 16 ks .. +15, all 256 head dims: MN-major B operand whose
+        // 64-wide head-dim slabs are kSlabK apart.
+        const uint64_t bd = umma_desc_sw128(kv_base + (j * kKB + ks * 16) * 128, kSlabK, 1024);
         umma_bf16(tO, ad, bd, idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
       }
-      umma_commit(&kv_empty[s]);
     }
     if (good) umma_commit(o_full);
   } else if (warp >= 2) {
@@ -199,79 +190,76 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
     const bool has_blk = g < nblk;
     const int key0 = (kb0 + g) * kKB;
-    // this thread's block of S (threads of absent blocks wait for the last block,
-    // which every thread needs before P may overwrite Q)
-    bool good = __all_sync(0xffffffffu, mbar_wait(&s_full[has_blk ? g : nblk - 1], 0, a.err,
-                                                  KERR_WAIT_MMA));
+    bool good = __all_sync(0xffffffffu, mbar_wait(s_full, 0, a.err, KERR_WAIT_MMA));
     tc_fence_after();
     float mx = -INFINITY, l = 0.f;
     const int nvis = min(kKB, max(0, limit - key0));
     const int p_rel = P - key0, lo_rel = P + lo - key0;  // hidden: p_rel <= i < lo_rel
-    uint4 pk[8];  // P of this block against the block's own max, bf16, logical order
+    // every key of the block visible (the common case): no per-key mask
+    const bool all_vis = nvis == kKB && (p_rel >= kKB || lo_rel <= 0);
+    uint32_t sv[64];
     if (good && has_blk) {
-      uint32_t sv[64];
       uint32_t (&s0)[32] = *reinterpret_cast<uint32_t(*)[32]>(&sv[0]);
       uint32_t (&s1)[32] = *reinterpret_cast<uint32_t(*)[32]>(&sv[32]);
       tmem_ld32_nowait(tS + lane_off + g * kKB, s0);
       tmem_ld32_nowait(tS + lane_off + g * kKB + 32, s1);
       tmem_ld_wait();
+      if (all_vis) {
+        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int i = 0; i < 64; ++i)
-        if (i < nvis && (i < p_rel || i >= lo_rel)) mx = fmaxf(mx, __uint_as_float(sv[i]));
-      const float mscaled = mx > -INFINITY ? mx * a.scale_log2 : 0.f;
+        for (int i = 0; i < 64; ++i) m4[i & 3] = fmaxf(m4[i & 3], __uint_as_float(sv[i]));
+        mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+      } else {
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {  // keys 8c .. 8c+7
-        float p[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int kk = c * 8 + i;
-          const float e = exp2f(fmaf(__uint_as_float(sv[kk]), a.scale_log2, -mscaled));
-          const bool vis = kk < nvis && (kk < p_rel || kk >= lo_rel);
-          const float pr = vis ? __bfloat162float(__float2bfloat16_rn(e)) : 0.f;
-          l += pr;
-          p[i] = pr;
-        }
-        pk[c] = pack_bf16x8(p);
+        for (int i = 0; i < 64; ++i)
+          if (i < nvis && (i < p_rel || i >= lo_rel)) mx = fmaxf(mx, __uint_as_float(sv[i]));
       }
     }
     xmax[g * kRows + row] = mx;
-    xsum[g * kRows + row] = l;
-    // block maxima and sums of every row.  The threads of the last block (and of
-    // absent blocks) waited for the last S commit, which covers every S MMA, so
-    // past this barrier Q is dead for all threads and P may go over it.
+    // S is complete (every thread waited for its commit), so past this barrier Q
+    // is dead for all threads and P may go over it
     softmax_bar();
-    float bm[kBlocksPerSplit];
+    float mrow = xmax[row];
 #pragma unroll
-    for (int j = 0; j < kBlocksPerSplit; ++j) bm[j] = xmax[j * kRows + row];
-    const float mrow = fmaxf(fmaxf(bm[0], bm[1]), fmaxf(bm[2], bm[3]));
-    // row sum over blocks, each block's sum scaled to the row max
-    l = 0.f;
-#pragma unroll
-    for (int j = 0; j < kBlocksPerSplit; ++j)
-      if (bm[j] > -INFINITY) l += xsum[j * kRows + row] * exp2f((bm[j] - mrow) * a.scale_log2);
+    for (int j = 1; j < kBlocksPerSplit; ++j) mrow = fmaxf(mrow, xmax[j * kRows + row]);
     if (good && has_blk) {
-      // P, rescaled to the row max, goes over Q, 128-byte swizzled
+      // P = exp(S - row max) over visible keys, rounded to bf16 (the row sum adds
+      // the rounded values the P V MMA uses), 128-byte swizzled over Q
+      const float mscaled = mrow > -INFINITY ? mrow * a.scale_log2 : 0.f;
       uint8_t* prow = sQP + g * (kRows * 128) + row * 128;
-      const float alpha = mx > -INFINITY ? exp2f((mx - mrow) * a.scale_log2) : 0.f;
+      float l2[2] = {0.f, 0.f};
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        uint4 u = pk[c];
-        if (alpha != 1.f) {
-          __nv_bfloat162* h2 = reinterpret_cast<__nv_bfloat162*>(&u);
+      for (int c = 0; c < 8; ++c) {  // keys 8c .. 8c+7
+        uint32_t w[4];
 #pragma unroll
-          for (int q2 = 0; q2 < 4; ++q2) {
-            const float2 f = __bfloat1622float2(h2[q2]);
-            h2[q2] = __floats2bfloat162_rn(f.x * alpha, f.y * alpha);
+        for (int i = 0; i < 8; i += 2) {
+          const int kk = c * 8 + i;
+          float e0 = ex2_approx(fmaf(__uint_as_float(sv[kk]), a.scale_log2, -mscaled));
+          float e1 = ex2_approx(fmaf(__uint_as_float(sv[kk + 1]), a.scale_log2, -mscaled));
+          if (!all_vis) {
+            if (!(kk < nvis && (kk < p_rel || kk >= lo_rel))) e0 = 0.f;
+            if (!(kk + 1 < nvis && (kk + 1 < p_rel || kk + 1 >= lo_rel))) e1 = 0.f;
           }
+          // P is the bf16 rounding; the row sum adds exactly those values
+          const __nv_bfloat162 b2 = __floats2bfloat162_rn(e0, e1);
+          w[i / 2] = *reinterpret_cast<const uint32_t*>(&b2);
+          l2[0] += __uint_as_float(w[i / 2] << 16);
+          l2[1] += __uint_as_float(w[i / 2] & 0xFFFF0000u);
         }
-        *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) * 16)) = u;
+        *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) * 16)) = make_uint4(w[0], w[1], w[2], w[3]);
       }
+      l = l2[0] + l2[1];
     }
+    xsum[g * kRows + row] = l;
     mx = mrow;
     fence_proxy_async_smem();
     mbar_arrive(p_full);
     if (good) good = __all_sync(0xffffffffu, mbar_wait(o_full, 0, a.err, KERR_WAIT_MMA));
     tc_fence_after();
+    softmax_bar();  // every block's sum is in xsum
+    l = 0.f;
+#pragma unroll
+    for (int j = 0; j < kBlocksPerSplit; ++j) l += xsum[j * kRows + row];
     const int gtile = r * a.tiles_per_req + tile;
     const int grow = qrow0 + row;  // global q row = (r*T + t) * nq + head
     const int c0 = g * 64;         // O columns of this thread
@@ -282,8 +270,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld32_nowait(tO + lane_off + c0, o0);
       tmem_ld32_nowait(tO + lane_off + c0 + 32, o1);
       tmem_ld_wait();
-      // P, Q and the K/V ring are dead once O is complete: each warp stages its
-      // 32 rows there for coalesced stores
+      // P, Q and K/V are dead once O is complete: each warp stages its 32 rows
+      // there for coalesced stores
       uint8_t* stage = smem + (warp - 2) * (32 * 144);
       // one split: the output row; several: this split's partial (O / l, with
       // max and sum) for attn_merge_kernel
@@ -303,6 +291,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (nsplit > 1 && valid && g == 0) __stcg(a.part_ml + prow_idx, make_float2(mx, l));
     }
   }
+  // the producer and MMA lanes rejoin their warps first: a CTA barrier reached
+  // by a split warp does not wait for the rest of the CTA
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {

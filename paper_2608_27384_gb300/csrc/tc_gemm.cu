@@ -134,6 +134,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       gemm_epilogue<BN, MODE>(ep, trow, m0 + row, M, n0, split, stage, lane);
     }
   }
+  // the producer and MMA lanes rejoin their warps first: a CTA barrier reached
+  // by a split warp does not wait for the rest of the CTA
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -284,6 +287,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(&acc_empty[buf]);
     }
   }
+  // the producer and MMA lanes rejoin their warps first: a CTA barrier reached
+  // by a split warp does not wait for the rest of the CTA
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
