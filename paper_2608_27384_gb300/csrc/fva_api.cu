@@ -151,6 +151,7 @@ struct fva_handle {
   int* prefix_len_dev = nullptr;
   std::vector<int> layer_len;  // [Bmax * L], -1 = never set
   float2* rope = nullptr;
+  uint32_t* rope_h = nullptr;  // fp16 copy for the bf16 QKV epilogue
   float2* temb_freq = nullptr;  // [W/2] two-float split of 2 / p_j
   // activations / scratch
   void *temb = nullptr, *t1 = nullptr, *cond = nullptr, *y = nullptr, *q = nullptr;
@@ -365,6 +366,7 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
   if ((st = dalloc(h, &h->kc, kv_elems, a)) || (st = dalloc(h, &h->vc, kv_elems, a)) ||
       (st = dalloc(h, &h->prefix_len_dev, h->Bmax)) ||
       (st = dalloc(h, &h->rope, (size_t)h->S_cap * (h->dh / 2))) ||
+      (st = dalloc(h, &h->rope_h, (size_t)h->S_cap * (h->dh / 2))) ||
       (st = dalloc(h, &h->temb, (size_t)h->BKmax * h->W, a)) ||
       (st = dalloc(h, &h->t1, (size_t)h->BKmax * h->W, a)) ||
       (st = dalloc(h, &h->cond, (size_t)h->BKmax * h->W, a)) ||
@@ -464,7 +466,7 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
       return fail(FVA_ERR_UNSUPPORTED, "n_chunks * action_dim too large for the final kernel");
     CUDA_TRY(final_init(d));
   }
-  launch_rope_table(h->rope, h->S_cap, h->dh, c.rope_theta, 0);
+  launch_rope_table(h->rope, h->rope_h, h->S_cap, h->dh, c.rope_theta, 0);
   CUDA_TRY(cudaGetLastError());
   {
     // 2 / p_j in half turns per unit tau, p_j = t_min (t_max / t_min)^(j / (W/2 - 1))
@@ -940,6 +942,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.vc = vc_l;
       ep.prefix_len = h->prefix_len_dev;
       ep.rope = h->rope;
+      ep.rope_h = h->rope_h;
       ep.T = h->T;
       ep.S_cap = h->S_cap;
       ep.nq = h->nq;
@@ -1016,6 +1019,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       eq.vc = (uint8_t*)h->vc + (size_t)(last ? l : l + 1) * kv_layer * a;
       eq.prefix_len = h->prefix_len_dev;
       eq.rope = h->rope;
+      eq.rope_h = h->rope_h;
       eq.T = h->T;
       eq.S_cap = h->S_cap;
       eq.nq = h->nq;

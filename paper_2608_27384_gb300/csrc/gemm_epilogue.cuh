@@ -4,6 +4,7 @@
 // block kernel.
 #pragma once
 
+#include <cuda_fp16.h>
 #include "common.cuh"
 #include "kernels.h"
 
@@ -34,6 +35,72 @@ __device__ __forceinline__ void gemm_epilogue_prefetch_rope(const GemmEpi& ep, i
   const char* p = reinterpret_cast<const char*>(ep.rope + (size_t)pos * (dh / 2) + tj * (BN / 2));
 #pragma unroll
   for (int b = 0; b < (BN / 2) * 8; b += 128) asm volatile("prefetch.global.L1 [%0];" ::"l"(p + b));
+}
+
+// This row's fp16 RoPE (cos, sin) pairs for tile column n0 (BN/2 pairs, 2*BN
+// bytes), loaded into registers while the MMAs still run; zeros where the row
+// is past M or the tile is not rotated (v).
+template <int BN>
+__device__ __forceinline__ void gemm_epilogue_load_rope(const GemmEpi& ep, int m, int M, int n0,
+                                                        uint4 (&rh)[BN / 8]) {
+  const int dh = ep.dh, seg = n0 / dh, tj = (n0 % dh) / BN;
+  const bool need = m < M && seg <= ep.nq;
+  int pos = 0;
+  if (need) {
+    const int r = m / ep.T;
+    pos = __ldg(ep.prefix_len + r) + (m - r * ep.T);
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(ep.rope_h + (size_t)pos * (dh / 2) + tj * (BN / 2));
+#pragma unroll
+  for (int i = 0; i < BN / 8; ++i) rh[i] = need ? __ldg(src + i) : make_uint4(0u, 0u, 0u, 0u);
+}
+
+// The QKV epilogue (GEMM_QKV_ROPE) with the row's RoPE pairs already in
+// registers (gemm_epilogue_load_rope).  Weight rows are permuted so that tile
+// column c < BN/2 holds head dim d = tj*BN/2 + c of segment `seg` and column
+// c + BN/2 holds its rotate-half partner d + dh/2.  Segments: q heads 0..nq-1,
+// then k, then v.
+template <int BN>
+__device__ __forceinline__ void gemm_epilogue_qkv(const GemmEpi& ep, uint32_t trow, int m, int M,
+                                                  int n0, uint8_t* stage, int lane,
+                                                  const uint4 (&rh)[BN / 8]) {
+  constexpr int half = BN / 2;
+  const bool ok = m < M;
+  const int dh = ep.dh, seg = n0 / dh, tj = (n0 % dh) / BN;
+  int r = 0, t = 0, pos = 0;
+  if (ok) {
+    r = m / ep.T;
+    t = m - r * ep.T;
+    pos = __ldg(ep.prefix_len + r) + t;
+  }
+  bf16* dst;
+  if (seg < ep.nq)
+    dst = (bf16*)ep.q + (size_t)m * ep.nq * dh + seg * dh;
+  else
+    dst = (bf16*)(seg == ep.nq ? ep.kc : ep.vc) + ((size_t)r * ep.S_cap + pos) * dh;
+  const bool rotate = seg <= ep.nq;
+  const __half2* hp = reinterpret_cast<const __half2*>(rh);
+#pragma unroll
+  for (int c = 0; c < half; c += 32) {
+    float x1[32], x2[32];
+    tmem_ld32(trow + c, x1);
+    tmem_ld32(trow + half + c, x2);
+    if (rotate) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const float2 cs = __half22float2(hp[c + i]);
+        const float a0 = x1[i], b0 = x2[i];
+        x1[i] = a0 * cs.x - b0 * cs.y;
+        x2[i] = b0 * cs.x + a0 * cs.y;
+      }
+    }
+    const int d0 = tj * half + c;
+    uint4 p1[4], p2[4];
+    pack_bf16x32(x1, p1);
+    pack_bf16x32(x2, p2);
+    warp_store_rows<64>(stage, p1, ok ? dst + d0 : nullptr, lane);
+    warp_store_rows<64>(stage, p2, ok ? dst + d0 + dh / 2 : nullptr, lane);
+  }
 }
 
 // Epilogue of one output row per thread; `stage` is this warp's private shared

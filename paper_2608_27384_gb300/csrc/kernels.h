@@ -71,7 +71,9 @@ cudaError_t gemv_init(int K);
 void launch_gemv_silu(const void* in, const void* w, const float* bias, void* out, int M, int N,
                       int K, cudaStream_t s);
 
-void launch_rope_table(float2* table, int n_pos, int dh, float theta, cudaStream_t s);
+// (cos, sin) of position x frequency for RoPE, fp32 and rounded to fp16 pairs.
+void launch_rope_table(float2* table, uint32_t* table_h, int n_pos, int dh, float theta,
+                       cudaStream_t s);
 
 void launch_to_f32(const void* src, bool src_bf16, float* dst, long long n, cudaStream_t s);
 
@@ -103,6 +105,7 @@ struct GemmEpi {
   void* vc;
   const int* prefix_len;
   const float2* rope;   // [n_pos, dh/2] (cos, sin)
+  const uint32_t* rope_h;  // the same table as fp16 (cos, sin) pairs
   int T, S_cap, nq, dh;
   int* err;
 };

@@ -2,6 +2,7 @@
 // in-projection + first FiLM RMSNorm, the fused split-K reduction + gated
 // residual + FiLM RMSNorm, and the fused final norm + out-projection + Euler
 // update + emit + buffer roll + tail noise.  Plus small table / debug helpers.
+#include <cuda_fp16.h>
 #include "common.cuh"
 #include "kernels.h"
 
@@ -583,25 +584,29 @@ void launch_gemv_silu(const void* in, const void* w, const float* bias, void* ou
 // ----------------------------------------------------------------------------
 // tables and debug helpers
 // ----------------------------------------------------------------------------
-__global__ void rope_table_kernel(float2* table, int n_pos, int dh, double theta) {
+__global__ void rope_table_kernel(float2* table, uint32_t* table_h, int n_pos, int dh,
+                                  double theta) {
   const int half = dh / 2;
   const long long n = (long long)n_pos * half;
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n;
        i += (long long)gridDim.x * blockDim.x) {
     const int pos = (int)(i / half), p = (int)(i % half);
-    if (theta == 0.0) {
-      table[i] = make_float2(1.f, 0.f);
-    } else {
+    float2 v = make_float2(1.f, 0.f);
+    if (theta != 0.0) {
       const double ang = (double)pos * pow(theta, -2.0 * (double)p / (double)dh);
       double sn, cs;
       sincos(ang, &sn, &cs);
-      table[i] = make_float2((float)cs, (float)sn);
+      v = make_float2((float)cs, (float)sn);
     }
+    table[i] = v;
+    const __half2 hv = __floats2half2_rn(v.x, v.y);
+    table_h[i] = *reinterpret_cast<const uint32_t*>(&hv);
   }
 }
 
-void launch_rope_table(float2* table, int n_pos, int dh, float theta, cudaStream_t s) {
-  rope_table_kernel<<<304, 256, 0, s>>>(table, n_pos, dh, (double)theta);
+void launch_rope_table(float2* table, uint32_t* table_h, int n_pos, int dh, float theta,
+                       cudaStream_t s) {
+  rope_table_kernel<<<304, 256, 0, s>>>(table, table_h, n_pos, dh, (double)theta);
 }
 
 __global__ void to_f32_kernel(const void* src, bool src_bf16, float* dst, long long n) {

@@ -123,7 +123,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------- epilogue: warp w reads TMEM lanes 32*(w%4) .. +31
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;
-    if constexpr (MODE == GEMM_QKV_ROPE) gemm_epilogue_prefetch_rope<BN>(ep, m0 + row, M, n0);
+    uint4 rh[MODE == GEMM_QKV_ROPE ? BN / 8 : 1];
+    if constexpr (MODE == GEMM_QKV_ROPE) gemm_epilogue_load_rope<BN>(ep, m0 + row, M, n0, rh);
     const bool good = __all_sync(0xffffffffu, mbar_wait(acc_full, 0, ep.err, KERR_WAIT_MMA));
     tc_fence_after();
     if (good && nkb > 0) {
@@ -131,7 +132,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       // first stage is free to stage this warp's coalesced stores
       const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
       uint8_t* stage = smem + (warp - 2) * (32 * 144);
-      gemm_epilogue<BN, MODE>(ep, trow, m0 + row, M, n0, split, stage, lane);
+      if constexpr (MODE == GEMM_QKV_ROPE)
+        gemm_epilogue_qkv<BN>(ep, trow, m0 + row, M, n0, stage, lane, rh);
+      else
+        gemm_epilogue<BN, MODE>(ep, trow, m0 + row, M, n0, split, stage, lane);
     }
   }
   // the producer and MMA lanes rejoin their warps first: a CTA barrier reached
