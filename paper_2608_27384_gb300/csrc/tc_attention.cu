@@ -85,8 +85,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* kv_full = bars + 1;   // [4]: key block b of K (phase 0), then of V (phase 1)
   uint64_t* k_free = bars + 5;    // the S MMAs have read K
   uint64_t* s_full = bars + 6;    // S is in TMEM
-  uint64_t* p_full = bars + 7;
-  uint64_t* o_full = bars + 8;
+  uint64_t* o_full = bars + 7;
+  uint64_t* p_full = bars + 8;    // [4]: P of key block b is in shared memory
   uint32_t* tmem_slot = (uint32_t*)(bars + 15);
   float* xmax = (float*)(bars + 128);   // [4][128] per-block row max
   float* xsum = xmax + 4 * kRows;       // [4][128] per-block row sum
@@ -97,7 +97,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int b = 0; b < kBlocksPerSplit; ++b) mbar_init(&kv_full[b], 1);
     mbar_init(k_free, 1);
     mbar_init(s_full, 1);
-    mbar_init(p_full, kSoftmaxThreads);
+    for (int b = 0; b < kBlocksPerSplit; ++b) mbar_init(&p_full[b], kSoftmaxThreads / 32);
     mbar_init(o_full, 1);
     fence_barrier_init();
     tma_prefetch_desc(&tmQ);
@@ -157,10 +157,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       umma_commit(k_free);
       umma_commit(s_full);
     }
-    if (good) good = mbar_wait(p_full, 0, a.err, KERR_WAIT_SYNC);
-    tc_fence_after();
     for (int j = 0; good && j < nblk; ++j) {
-      if (!mbar_wait(&kv_full[j], 1, a.err, KERR_WAIT_TMA)) {
+      // block j's P (written while the softmax threads still work on later
+      // blocks) and V
+      if (!mbar_wait(&p_full[j], 0, a.err, KERR_WAIT_SYNC) ||
+          !mbar_wait(&kv_full[j], 1, a.err, KERR_WAIT_TMA)) {
         good = false;
         break;
       }
@@ -176,8 +177,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (good) umma_commit(o_full);
   } else if (warp >= 2) {
-    // ---------------- softmax + epilogue: thread (key block g, row)
-    const int g = (warp - 2) >> 2;          // key block of S / 64 dh columns of O
+    // ---------------- softmax + epilogue: thread (key quarter g, row) takes
+    // keys 16g .. 16g+15 of every key block, block after block, so that block
+    // j's P is complete (and its P V MMAs can start) while later blocks are
+    // still being exponentiated; in the epilogue it takes O columns 64g .. +63.
+    const int g = (warp - 2) >> 2;
     const int quarter = warp & 3;
     const int row = quarter * 32 + lane;
     const int t = t0 + row / a.nq;
@@ -188,31 +192,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int pad = a.pad_tokens ? __ldg(a.pad_tokens + r) : 0;
     const int lo = a.block_diag && valid ? max(pad, (t / a.H) * a.H) : pad;
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    const bool has_blk = g < nblk;
-    const int key0 = (kb0 + g) * kKB;
     bool good = __all_sync(0xffffffffu, mbar_wait(s_full, 0, a.err, KERR_WAIT_MMA));
     tc_fence_after();
-    float mx = -INFINITY, l = 0.f;
-    const int nvis = min(kKB, max(0, limit - key0));
-    const int p_rel = P - key0, lo_rel = P + lo - key0;  // hidden: p_rel <= i < lo_rel
-    // every key of the block visible (the common case): no per-key mask
-    const bool all_vis = nvis == kKB && (p_rel >= kKB || lo_rel <= 0);
-    uint32_t sv[64];
-    if (good && has_blk) {
-      uint32_t (&s0)[32] = *reinterpret_cast<uint32_t(*)[32]>(&sv[0]);
-      uint32_t (&s1)[32] = *reinterpret_cast<uint32_t(*)[32]>(&sv[32]);
-      tmem_ld32_nowait(tS + lane_off + g * kKB, s0);
-      tmem_ld32_nowait(tS + lane_off + g * kKB + 32, s1);
+    // visible keys of block j for this thread: i < nv[j] and not p_rel <= i < lo_rel
+    auto key_vis = [&](int j, int i) {
+      const int key = (kb0 + j) * kKB + g * 16 + i;
+      return key < limit && (key < P || key >= P + lo);
+    };
+    auto block_all_vis = [&](int j) {
+      const int k0 = (kb0 + j) * kKB + g * 16;
+      return k0 + 16 <= limit && (k0 + 16 <= P || k0 >= P + lo);
+    };
+    float mx = -INFINITY;
+    uint32_t sv[kBlocksPerSplit][16];
+    if (good) {
+#pragma unroll
+      for (int j = 0; j < kBlocksPerSplit; ++j)
+        if (j < nblk) tmem_ld16_nowait(tS + lane_off + j * kKB + g * 16, sv[j]);
       tmem_ld_wait();
-      if (all_vis) {
-        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-        for (int i = 0; i < 64; ++i) m4[i & 3] = fmaxf(m4[i & 3], __uint_as_float(sv[i]));
-        mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
-      } else {
+      for (int j = 0; j < kBlocksPerSplit; ++j) {
+        if (j >= nblk) break;
+        if (block_all_vis(j)) {
 #pragma unroll
-        for (int i = 0; i < 64; ++i)
-          if (i < nvis && (i < p_rel || i >= lo_rel)) mx = fmaxf(mx, __uint_as_float(sv[i]));
+          for (int i = 0; i < 16; ++i) mx = fmaxf(mx, __uint_as_float(sv[j][i]));
+        } else {
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            if (key_vis(j, i)) mx = fmaxf(mx, __uint_as_float(sv[j][i]));
+        }
       }
     }
     xmax[g * kRows + row] = mx;
@@ -222,41 +230,45 @@ __global__ void __launch_bounds__(kThreads, 1)
     float mrow = xmax[row];
 #pragma unroll
     for (int j = 1; j < kBlocksPerSplit; ++j) mrow = fmaxf(mrow, xmax[j * kRows + row]);
-    if (good && has_blk) {
-      // P = exp(S - row max) over visible keys, rounded to bf16 (the row sum adds
-      // the rounded values the P V MMA uses), 128-byte swizzled over Q
-      const float mscaled = mrow > -INFINITY ? mrow * a.scale_log2 : 0.f;
-      uint8_t* prow = sQP + g * (kRows * 128) + row * 128;
-      float l2[2] = {0.f, 0.f};
+    const float mscaled = mrow > -INFINITY ? mrow * a.scale_log2 : 0.f;
+    float l2[2] = {0.f, 0.f};
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {  // keys 8c .. 8c+7
-        uint32_t w[4];
+    for (int j = 0; j < kBlocksPerSplit; ++j) {
+      if (j >= nblk) break;
+      if (good) {
+        // P = exp(S - row max) over visible keys, rounded to bf16 (the row sum
+        // adds the rounded values the P V MMA uses), 128-byte swizzled over Q
+        const bool all_vis = block_all_vis(j);
+        uint32_t w[8];
 #pragma unroll
-        for (int i = 0; i < 8; i += 2) {
-          const int kk = c * 8 + i;
-          float e0 = ex2_approx(fmaf(__uint_as_float(sv[kk]), a.scale_log2, -mscaled));
-          float e1 = ex2_approx(fmaf(__uint_as_float(sv[kk + 1]), a.scale_log2, -mscaled));
+        for (int i = 0; i < 16; i += 2) {
+          float e0 = ex2_approx(fmaf(__uint_as_float(sv[j][i]), a.scale_log2, -mscaled));
+          float e1 = ex2_approx(fmaf(__uint_as_float(sv[j][i + 1]), a.scale_log2, -mscaled));
           if (!all_vis) {
-            if (!(kk < nvis && (kk < p_rel || kk >= lo_rel))) e0 = 0.f;
-            if (!(kk + 1 < nvis && (kk + 1 < p_rel || kk + 1 >= lo_rel))) e1 = 0.f;
+            if (!key_vis(j, i)) e0 = 0.f;
+            if (!key_vis(j, i + 1)) e1 = 0.f;
           }
-          // P is the bf16 rounding; the row sum adds exactly those values
           const __nv_bfloat162 b2 = __floats2bfloat162_rn(e0, e1);
           w[i / 2] = *reinterpret_cast<const uint32_t*>(&b2);
           l2[0] += __uint_as_float(w[i / 2] << 16);
           l2[1] += __uint_as_float(w[i / 2] & 0xFFFF0000u);
         }
-        *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) * 16)) = make_uint4(w[0], w[1], w[2], w[3]);
+        uint8_t* prow = sQP + j * (kRows * 128) + row * 128;
+        *reinterpret_cast<uint4*>(prow + (((2 * g) ^ (row & 7)) * 16)) =
+            make_uint4(w[0], w[1], w[2], w[3]);
+        *reinterpret_cast<uint4*>(prow + (((2 * g + 1) ^ (row & 7)) * 16)) =
+            make_uint4(w[4], w[5], w[6], w[7]);
       }
-      l = l2[0] + l2[1];
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[j]);
     }
+    float l = l2[0] + l2[1];
     xsum[g * kRows + row] = l;
     mx = mrow;
-    fence_proxy_async_smem();
-    mbar_arrive(p_full);
     if (good) good = __all_sync(0xffffffffu, mbar_wait(o_full, 0, a.err, KERR_WAIT_MMA));
     tc_fence_after();
-    softmax_bar();  // every block's sum is in xsum
+    softmax_bar();  // every quarter's sum is in xsum
     l = 0.f;
 #pragma unroll
     for (int j = 0; j < kBlocksPerSplit; ++j) l += xsum[j * kRows + row];
