@@ -1050,13 +1050,13 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.ldo = W;
       ep.split_stride = pstride;
       mark(FVA_K_OUT_PROJ, l);
-      CUDA_TRY(launch_tc_gemm(kBnResid, GEMM_PARTIAL_F32, &h->m_attn, &lw.m_o, ep, M, W, Dq, sp_o, s));
+      CUDA_TRY(launch_tc_gemm(kBnResid, GEMM_PARTIAL_BF16, &h->m_attn, &lw.m_o, ep, M, W, Dq, sp_o, s));
     } else {
       launch_f32_gemm((float*)h->attn, Dq, (float*)lw.w_o, h->part, W, M, W, Dq, s);
     }
     mark(FVA_K_RESID_NORM, l);
-    launch_resid_norm(d, h->h, h->part, sp_o, pstride, h->mod, mod_off(l, 2, W), mod_off(l, 3, W),
-                      mod_off(l, 4, W), h->y, bf, s);
+    launch_resid_norm(d, h->h, h->part, bf, sp_o, pstride, h->mod, mod_off(l, 2, W),
+                      mod_off(l, 3, W), mod_off(l, 4, W), h->y, bf, s);
     if (trace) {
       CUDA_TRY(copy_h(o_hmid));
       launch_to_f32(h->y, bf, tr_at(o_y2), (long long)MW, s);
@@ -1073,7 +1073,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.ldo = W;
       ep.split_stride = pstride;
       mark(FVA_K_DOWN, l);
-      CUDA_TRY(launch_tc_gemm(kBnResid, GEMM_PARTIAL_F32, &h->m_mlp, &lw.m_d, ep, M, W, F, sp_d, s));
+      CUDA_TRY(launch_tc_gemm(kBnResid, GEMM_PARTIAL_BF16, &h->m_mlp, &lw.m_d, ep, M, W, F, sp_d, s));
     } else {
       launch_f32_gemm((float*)h->y, W, (float*)lw.w_gu, h->c32, 2 * F, M, 2 * F, W, s);
       launch_f32_geglu(h->c32, (float*)h->mlp, M, F, s);
@@ -1082,7 +1082,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     if (trace) launch_to_f32(h->mlp, bf, tr_at(o_mlp), (long long)M * F, s);
     if (l + 1 < L) {
       mark(FVA_K_RESID_NORM, l);
-      launch_resid_norm(d, h->h, h->part, sp_d, pstride, h->mod, mod_off(l, 5, W),
+      launch_resid_norm(d, h->h, h->part, bf, sp_d, pstride, h->mod, mod_off(l, 5, W),
                         mod_off(l + 1, 0, W), mod_off(l + 1, 1, W), h->y, bf, s);
       if (trace) CUDA_TRY(copy_h(o_hout));
     }
@@ -1090,7 +1090,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   // ---- final norm, out-projection, Euler update, emit, roll, tail
   if (!blk) {
     mark(FVA_K_FINAL, -1);
-    launch_final_norm(d, h->h, h->part, sp_d, pstride, h->mod, h->yF, s);
+    launch_final_norm(d, h->h, h->part, bf, sp_d, pstride, h->mod, h->yF, s);
   }
   mark(FVA_K_VELOCITY, -1);
   launch_velocity_euler(d, h->yF, h->w_out_t, h->b_out, h->dt_dev(), buffer, out_chunk, h->vel,

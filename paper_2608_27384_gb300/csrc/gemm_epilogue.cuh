@@ -111,8 +111,19 @@ template <int BN, int MODE>
 __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, int m, int M,
                                               int n0, int split, uint8_t* stage, int lane) {
   const bool ok = m < M;
-  if constexpr (MODE == GEMM_BIAS_F32 || MODE == GEMM_BIAS_SILU_BF16 ||
-                MODE == GEMM_PARTIAL_F32) {
+  if constexpr (MODE == GEMM_PARTIAL_BF16) {
+#pragma unroll 1
+    for (int c = 0; c < BN; c += 32) {
+      float v[32];
+      tmem_ld32(trow + c, v);
+      uint4 u[4];
+      pack_bf16x32(v, u);
+      bf16* dst = ok ? (bf16*)ep.out + split * ep.split_stride + (size_t)m * ep.ldo + n0 + c
+                     : nullptr;
+      warp_store_rows<64>(stage, u, dst, lane);
+    }
+  } else if constexpr (MODE == GEMM_BIAS_F32 || MODE == GEMM_BIAS_SILU_BF16 ||
+                       MODE == GEMM_PARTIAL_F32) {
 #pragma unroll 1
     for (int c = 0; c < BN; c += 32) {
       float v[32];

@@ -49,17 +49,18 @@ void launch_embed_norm(const StepDims& d, const float* buffer, const float* w_in
                        int n_sms, cudaStream_t s);
 
 // h += gate * sum_z part[z];  y = rmsnorm(h) * (1 + scale) + shift.
-void launch_resid_norm(const StepDims& d, float* h, const float* part, int n_parts,
-                       long long part_stride, const float* mod, int gate_off, int scale_off,
-                       int shift_off, void* y, bool act_bf16, cudaStream_t s);
+void launch_resid_norm(const StepDims& d, float* h, const void* part, bool part_bf16,
+                       int n_parts, long long part_stride, const float* mod, int gate_off,
+                       int scale_off, int shift_off, void* y, bool act_bf16, cudaStream_t s);
 
 // Final residual + final FiLM RMSNorm (fp32 y_F into yF [B*K*H, W]), then
 // out-projection, Euler update, emit, roll and tail (two launches).  w_out_t is
 // W_out transposed, [W, A] fp32.  final_init sets the second kernel's
 // shared-memory limit for these dimensions (once per handle).
 cudaError_t final_init(const StepDims& d);
-void launch_final_norm(const StepDims& d, float* h, const float* part, int n_parts,
-                       long long part_stride, const float* mod, float* yF, cudaStream_t s);
+void launch_final_norm(const StepDims& d, float* h, const void* part, bool part_bf16,
+                       int n_parts, long long part_stride, const float* mod, float* yF,
+                       cudaStream_t s);
 void launch_velocity_euler(const StepDims& d, const float* yF, const float* w_out_t,
                            const float* b_out, const float* dt, float* buffer, float* out_chunk,
                            float* vel_out, const float* fresh, unsigned long long seed,
@@ -92,6 +93,7 @@ enum GemmMode {
   GEMM_PARTIAL_F32 = 2,   // out f32 [split] = acc (split-K partial plane)
   GEMM_QKV_ROPE = 3,      // RoPE, q -> q buffer, k/v -> KV workspace (permuted weights)
   GEMM_GEGLU = 4,         // out bf16 = gelu(gate) * up (interleaved weights)
+  GEMM_PARTIAL_BF16 = 5,  // out bf16 [split] = acc (split-K partial plane)
 };
 
 struct GemmEpi {

@@ -216,9 +216,19 @@ void launch_embed_norm(const StepDims& d, const float* buffer, const float* w_in
 // h += gate_c * sum_z part[z]  (split-K partials reduced in fixed order z = 0..),
 // then y = FiLM RMSNorm(h) with the next norm's (scale, shift).  One CTA per row.
 // ----------------------------------------------------------------------------
-template <typename Act>
+// 4 consecutive partial-sum values as floats (fp32 or bf16 planes), L2 only.
+__device__ __forceinline__ float4 load4_cg(const float* p) {
+  return __ldcg(reinterpret_cast<const float4*>(p));
+}
+__device__ __forceinline__ float4 load4_cg(const bf16* p) {
+  const uint2 u = __ldcg(reinterpret_cast<const uint2*>(p));
+  return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xFFFF0000u),
+                     __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xFFFF0000u));
+}
+
+template <typename Act, typename Part>
 __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
-                                  const float* __restrict__ part, int n_parts,
+                                  const Part* __restrict__ part, int n_parts,
                                   long long part_stride, const float* __restrict__ mod,
                                   int gate_off, int scale_off, int shift_off,
                                   Act* __restrict__ y) {
@@ -236,7 +246,7 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
 #pragma unroll
     for (int z = 0; z < 8; ++z)
       if (z < n_parts)
-        p[z] = __ldcg(reinterpret_cast<const float4*>(part + z * part_stride + (size_t)m * d.W + col));
+        p[z] = load4_cg(part + z * part_stride + (size_t)m * d.W + col);
     const float4 g = *reinterpret_cast<const float4*>(mrow + gate_off + col);
     const float4 sc = *reinterpret_cast<const float4*>(mrow + scale_off + col);
     const float4 sh = *reinterpret_cast<const float4*>(mrow + shift_off + col);
@@ -248,7 +258,7 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
         acc.x += p[z].x; acc.y += p[z].y; acc.z += p[z].z; acc.w += p[z].w;
       }
     for (int z = 8; z < n_parts; ++z) {
-      const float4 q = __ldcg(reinterpret_cast<const float4*>(part + z * part_stride + (size_t)m * d.W + col));
+      const float4 q = load4_cg(part + z * part_stride + (size_t)m * d.W + col);
       acc.x += q.x; acc.y += q.y; acc.z += q.z; acc.w += q.w;
     }
     hv.x = fmaf(g.x, acc.x, hv.x);
@@ -265,10 +275,9 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
   }
   float ss = 0.f;
   for (int cc = col; cc < d.W; cc += blockDim.x * 4) {
-    float4 acc = __ldcg(reinterpret_cast<const float4*>(part + (size_t)m * d.W + cc));
+    float4 acc = load4_cg(part + (size_t)m * d.W + cc);
     for (int z = 1; z < n_parts; ++z) {
-      const float4 q =
-          __ldcg(reinterpret_cast<const float4*>(part + z * part_stride + (size_t)m * d.W + cc));
+      const float4 q = load4_cg(part + z * part_stride + (size_t)m * d.W + cc);
       acc.x += q.x; acc.y += q.y; acc.z += q.z; acc.w += q.w;
     }
     const float4 g = *reinterpret_cast<const float4*>(mrow + gate_off + cc);
@@ -285,17 +294,30 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
                           y + (size_t)m * d.W);
 }
 
-void launch_resid_norm(const StepDims& d, float* h, const float* part, int n_parts,
-                       long long part_stride, const float* mod, int gate_off, int scale_off,
-                       int shift_off, void* y, bool act_bf16, cudaStream_t s) {
+template <typename Part>
+static void launch_resid_norm_t(const StepDims& d, int rows, float* h, const Part* part,
+                                int n_parts, long long part_stride, const float* mod,
+                                int gate_off, int scale_off, int shift_off, void* y,
+                                bool act_bf16, cudaStream_t s) {
+  if (act_bf16)
+    launch_pdl(resid_norm_kernel<bf16, Part>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h,
+               part, n_parts, part_stride, mod, gate_off, scale_off, shift_off, (bf16*)y);
+  else
+    launch_pdl(resid_norm_kernel<float, Part>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h,
+               part, n_parts, part_stride, mod, gate_off, scale_off, shift_off, (float*)y);
+}
+
+void launch_resid_norm(const StepDims& d, float* h, const void* part, bool part_bf16,
+                       int n_parts, long long part_stride, const float* mod, int gate_off,
+                       int scale_off, int shift_off, void* y, bool act_bf16, cudaStream_t s) {
   const int rows = d.B * d.T;
   if (rows <= 0) return;
-  if (act_bf16)
-    launch_pdl(resid_norm_kernel<bf16>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h, part,
-               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (bf16*)y);
+  if (part_bf16)
+    launch_resid_norm_t(d, rows, h, (const bf16*)part, n_parts, part_stride, mod, gate_off,
+                        scale_off, shift_off, y, act_bf16, s);
   else
-    launch_pdl(resid_norm_kernel<float>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h, part,
-               n_parts, part_stride, mod, gate_off, scale_off, shift_off, (float*)y);
+    launch_resid_norm_t(d, rows, h, (const float*)part, n_parts, part_stride, mod, gate_off,
+                        scale_off, shift_off, y, act_bf16, s);
 }
 
 // ----------------------------------------------------------------------------
@@ -474,9 +496,10 @@ cudaError_t final_init(const StepDims& d) {
                               (int)vel_smem_bytes(d));
 }
 
-void launch_final_norm(const StepDims& d, float* h, const float* part, int n_parts,
-                       long long part_stride, const float* mod, float* yF, cudaStream_t s) {
-  launch_resid_norm(d, h, part, n_parts, part_stride, mod, mod_off(d.L - 1, 5, d.W),
+void launch_final_norm(const StepDims& d, float* h, const void* part, bool part_bf16,
+                       int n_parts, long long part_stride, const float* mod, float* yF,
+                       cudaStream_t s) {
+  launch_resid_norm(d, h, part, part_bf16, n_parts, part_stride, mod, mod_off(d.L - 1, 5, d.W),
                     modf_off(d.L, 0, d.W), modf_off(d.L, 1, d.W), yF, false, s);
 }
 

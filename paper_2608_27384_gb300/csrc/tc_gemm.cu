@@ -331,6 +331,7 @@ cudaError_t tc_gemm_init() {
   if ((e = set_attr<kBnFilm, GEMM_BIAS_F32>()) != cudaSuccess) return e;
   if ((e = set_attr<kBnQKV, GEMM_QKV_ROPE>()) != cudaSuccess) return e;
   if ((e = set_attr<kBnResid, GEMM_PARTIAL_F32>()) != cudaSuccess) return e;
+  if ((e = set_attr<kBnResid, GEMM_PARTIAL_BF16>()) != cudaSuccess) return e;
   if ((e = set_attr<kBnGU, GEMM_GEGLU>()) != cudaSuccess) return e;
   return cudaSuccess;
 }
@@ -347,6 +348,8 @@ cudaError_t launch_tc_gemm(int bn, int mode, const CUtensorMap* a, const CUtenso
     return launch<kBnQKV, GEMM_QKV_ROPE>(a, b, ep, M, N, K, splits, s);
   if (bn == kBnResid && mode == GEMM_PARTIAL_F32)
     return launch<kBnResid, GEMM_PARTIAL_F32>(a, b, ep, M, N, K, splits, s);
+  if (bn == kBnResid && mode == GEMM_PARTIAL_BF16)
+    return launch<kBnResid, GEMM_PARTIAL_BF16>(a, b, ep, M, N, K, splits, s);
   if (bn == kBnGU && mode == GEMM_GEGLU)
     return launch<kBnGU, GEMM_GEGLU>(a, b, ep, M, N, K, splits, s);
   return cudaErrorInvalidValue;
