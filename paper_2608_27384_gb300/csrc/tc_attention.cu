@@ -81,20 +81,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* sQP = smem;                      // 4 slabs [128 rows x 128 B]: Q, then P
   uint8_t* sKV = smem + kQBytes;            // 4 slabs [256 keys x 128 B]: K, then V
   uint64_t* bars = (uint64_t*)(sKV + kBlocksPerSplit * kKVBytes);
-  uint64_t* q_full = bars + 0;
-  uint64_t* kv_full = bars + 1;   // [4]: key block b of K (phase 0), then of V (phase 1)
-  uint64_t* k_free = bars + 5;    // the S MMAs have read K
-  uint64_t* s_full = bars + 6;    // S is in TMEM
-  uint64_t* o_full = bars + 7;
-  uint64_t* p_full = bars + 8;    // [4]: P of key block b is in shared memory
+  uint64_t* qk_full = bars + 0;   // [4]: head-dim slab j of Q and of every K block
+  uint64_t* v_full = bars + 4;    // [4]: V of key block b
+  uint64_t* k_free = bars + 8;    // the S MMAs have read K
+  uint64_t* s_full = bars + 9;    // S is in TMEM
+  uint64_t* o_full = bars + 10;
+  uint64_t* p_full = bars + 11;   // [4]: P of key block b is in shared memory
   uint32_t* tmem_slot = (uint32_t*)(bars + 15);
   float* xmax = (float*)(bars + 128);   // [4][128] per-block row max
   float* xsum = xmax + 4 * kRows;       // [4][128] per-block row sum
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    mbar_init(q_full, 1);
-    for (int b = 0; b < kBlocksPerSplit; ++b) mbar_init(&kv_full[b], 1);
+    for (int j = 0; j < 4; ++j) mbar_init(&qk_full[j], nblk + 1);  // Q slab + each K block's slab
+    for (int b = 0; b < kBlocksPerSplit; ++b) mbar_init(&v_full[b], 1);
     mbar_init(k_free, 1);
     mbar_init(s_full, 1);
     for (int b = 0; b < kBlocksPerSplit; ++b) mbar_init(&p_full[b], kSoftmaxThreads / 32);
@@ -122,38 +122,53 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Key blocks that lie wholly inside the prefix come from fva_set_prefix_kv,
     // not from the predecessor grid, so they are requested before waiting for
     // it; q and the action keys/values (written by the QKV projection) after.
-    // Every other thread only runs behind these loads.
-    auto load_block = [&](const CUtensorMap* map, int b) {
-      mbar_arrive_expect_tx(&kv_full[b], kKVBytes);
-      for (int j = 0; j < 4; ++j)
-        tma_load_2d(sKV + j * (kBlocksPerSplit * kKB * 128) + b * (kKB * 128), map, j * 64,
-                    krow0 + b * kKB, &kv_full[b]);
+    // Loads go out head-dim slab by slab, so the S MMAs of slab 0 can start
+    // while later slabs are in flight.  Every other thread only runs behind
+    // these loads.
+    constexpr uint32_t kSlab = kBlocksPerSplit * kKB * 128;
+    auto load_k = [&](int j, int b) {
+      mbar_arrive_expect_tx(&qk_full[j], kKB * 128);
+      tma_load_2d(sKV + j * kSlab + b * (kKB * 128), &tmK, j * 64, krow0 + b * kKB, &qk_full[j]);
     };
-    int b = 0;
-    for (; b < nblk && (kb0 + b + 1) * kKB <= P; ++b) load_block(&tmK, b);
+    int npre = 0;
+    while (npre < nblk && (kb0 + npre + 1) * kKB <= P) ++npre;
+    for (int j = 0; j < 4; ++j)
+      for (int b = 0; b < npre; ++b) load_k(j, b);
     pdl_wait();
-    mbar_arrive_expect_tx(q_full, kQBytes);
-    for (int j = 0; j < 4; ++j) tma_load_2d(sQP + j * (kRows * 128), &tmQ, j * 64, qrow0, q_full);
-    for (; b < nblk; ++b) load_block(&tmK, b);
+    for (int j = 0; j < 4; ++j) {
+      mbar_arrive_expect_tx(&qk_full[j], kRows * 128);
+      tma_load_2d(sQP + j * (kRows * 128), &tmQ, j * 64, qrow0, &qk_full[j]);
+      for (int b = npre; b < nblk; ++b) load_k(j, b);
+    }
     if (mbar_wait(k_free, 0, a.err, KERR_WAIT_MMA))
-      for (b = 0; b < nblk; ++b) load_block(&tmV, b);
+      for (int b = 0; b < nblk; ++b) {
+        mbar_arrive_expect_tx(&v_full[b], kKVBytes);
+        for (int j = 0; j < 4; ++j)
+          tma_load_2d(sKV + j * kSlab + b * (kKB * 128), &tmV, j * 64, krow0 + b * kKB,
+                      &v_full[b]);
+      }
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer
     const uint32_t idesc_s = umma_idesc_bf16(kRows, nblk * kKB, false);
     constexpr uint32_t idesc_o = umma_idesc_bf16(kRows, kDH, true);
     constexpr uint32_t kSlabK = kBlocksPerSplit * kKB * 128;  // 32 KB between head-dim slabs
-    bool good = mbar_wait(q_full, 0, a.err, KERR_WAIT_TMA);
-    for (int b = 0; good && b < nblk; ++b) good = mbar_wait(&kv_full[b], 0, a.err, KERR_WAIT_TMA);
-    tc_fence_after();
     const uint32_t qp_base = smem_u32(sQP), kv_base = smem_u32(sKV);
-    if (good) {
-#pragma unroll
-      for (int ks = 0; ks < kDH / 16; ++ks) {
-        const uint32_t off = (ks & 3) * 32;  // 16 bf16 along K inside the 128-byte row
-        const uint64_t ad = umma_desc_sw128(qp_base + (ks >> 2) * (kRows * 128) + off, 16, 1024);
-        const uint64_t bd = umma_desc_sw128(kv_base + (ks >> 2) * kSlabK + off, 16, 1024);
-        umma_bf16(tS, ad, bd, idesc_s, ks > 0 ? 1u : 0u);
+    bool good = true;
+    for (int j = 0; good && j < 4; ++j) {  // head-dim slab j: 4 steps of 16
+      if (!mbar_wait(&qk_full[j], 0, a.err, KERR_WAIT_TMA)) {
+        good = false;
+        break;
       }
+      tc_fence_after();
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        const uint32_t off = kk * 32;  // 16 bf16 along K inside the 128-byte row
+        const uint64_t ad = umma_desc_sw128(qp_base + j * (kRows * 128) + off, 16, 1024);
+        const uint64_t bd = umma_desc_sw128(kv_base + j * kSlabK + off, 16, 1024);
+        umma_bf16(tS, ad, bd, idesc_s, (j > 0 || kk > 0) ? 1u : 0u);
+      }
+    }
+    if (good) {
       umma_commit(k_free);
       umma_commit(s_full);
     }
@@ -161,7 +176,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // block j's P (written while the softmax threads still work on later
       // blocks) and V
       if (!mbar_wait(&p_full[j], 0, a.err, KERR_WAIT_SYNC) ||
-          !mbar_wait(&kv_full[j], 1, a.err, KERR_WAIT_TMA)) {
+          !mbar_wait(&v_full[j], 0, a.err, KERR_WAIT_TMA)) {
         good = false;
         break;
       }

@@ -25,6 +25,7 @@ def errors(got, ref):
 def assert_close(got, ref, max_abs=None, rel_l2=None, what=""):
     ma, rl = errors(got, ref)
     msg = f"{what}: max_abs={ma:.3e} rel_l2={rl:.3e}"
+    print(msg)  # the measured errors, shown with pytest -s / -rP
     if max_abs is not None:
         assert ma <= max_abs, msg
     if rel_l2 is not None:
