@@ -256,9 +256,21 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 // ----------------------------------------------------------------------------
 __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
 
+// 2^x by the PTX ex2.approx.ftz.f32 instruction (relative error about 2^-22;
+// results below 2^-126 flush to 0).
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// GELU, tanh form: 0.5 x (1 + tanh(u)) with u = sqrt(2/pi) (x + 0.044715 x^3),
+// evaluated as the identical x / (1 + e^(-2u)) (one exp2 and one fast divide;
+// for u below about -44 the exp2 overflows and the result is -0).
 __device__ __forceinline__ float gelu_tanh_f(float x) {
   const float k0 = 0.7978845608028654f;  // sqrt(2 / pi)
-  return 0.5f * x * (1.0f + tanhf(k0 * (x + 0.044715f * x * x * x)));
+  const float u = k0 * fmaf(0.044715f * x, x * x, x);
+  return __fdividef(x, 1.0f + ex2_approx(-2.8853900817779268f * u));  // -2 log2(e) u
 }
 
 __device__ __forceinline__ float warp_sum(float v) {

@@ -45,14 +45,6 @@ constexpr int kSmem = kQBytes + kBlocksPerSplit * kKVBytes + 1024 /*align*/ + 10
                       8 * kRows * 4 /*row exchange*/;
 constexpr uint32_t kTmemCols = 512;
 
-// 2^x by the PTX ex2.approx.ftz.f32 instruction (relative error about 2^-22,
-// far below the bf16 rounding P gets next; results below 2^-126 flush to 0)
-__device__ __forceinline__ float ex2_approx(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
 __device__ __forceinline__ void softmax_bar() {
   asm volatile("bar.sync 1, 512;" ::: "memory");
 }
