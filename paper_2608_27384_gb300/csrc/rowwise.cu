@@ -356,11 +356,14 @@ __device__ __forceinline__ float tail_normal(unsigned long long seed, unsigned l
 
 // ----------------------------------------------------------------------------
 // Velocity, Euler update, emit, roll and tail.  The final FiLM RMSNorm has
-// already written y_F [B*K*H, W] (fp32).  One CTA per (token position j within
-// a chunk, request r) owns column j of every chunk of request r, so the
-// in-place roll of the buffer is race-free.  The K rows of y_F and (a slice of)
-// W_out^T [W, A] are staged in shared memory with all loads in flight at once;
-// thread (k, a) then computes v[k][a] = b_out[a] + sum_w y_F[k][w] W_out^T[w][a].
+// already written y_F [B*K*H, W] (fp32).  A cluster of `nsplit` CTAs per (token
+// position j within a chunk, request r) owns column j of every chunk of request
+// r; CTA q of the cluster takes the width range [q W/nsplit, (q+1) W/nsplit).
+// Each stages its slice of the K rows of y_F and of W_out^T [W, A] in shared
+// memory with all loads in flight at once and forms the partial sums
+// v_q[k][a] = sum_w y_F[k][w] W_out^T[w][a] over its range; CTA 0 adds b_out[a]
+// and the partials in the order q = 0, 1, ... through distributed shared memory
+// and alone writes the buffer column, so the in-place roll is race-free.
 // x'_k = x_k + dt_k v_k (fp32, separately rounded multiply and add), out = x'_1,
 // slot k <- x'_{k+1}, tail <- z.
 // ----------------------------------------------------------------------------
@@ -372,10 +375,12 @@ __global__ void __launch_bounds__(kVelThreads)
                           const float* __restrict__ dt, float* __restrict__ buffer,
                           float* __restrict__ out_chunk, float* __restrict__ vel_out,
                           const float* __restrict__ fresh, unsigned long long seed,
-                          const unsigned long long* __restrict__ step_idx, int wchunk) {
+                          const unsigned long long* __restrict__ step_idx, int wchunk,
+                          int nsplit) {
   extern __shared__ __align__(16) float sm[];
   __shared__ __align__(8) uint64_t bar;
-  const int j = blockIdx.x, r = blockIdx.y;
+  const int q = blockIdx.x, j = blockIdx.y, r = blockIdx.z;  // q: rank in the cluster
+  const int wq = d.W / nsplit, wbeg = q * wq;
   const int KA = d.K * d.A;
   float* ys = sm;                    // [K][wchunk]
   float* ws = ys + d.K * wchunk;     // [wchunk][A]
@@ -392,11 +397,11 @@ __global__ void __launch_bounds__(kVelThreads)
   const size_t slot = (size_t)d.H * d.A;
   const float* xcol = buffer + ((size_t)r * d.K * d.H + j) * d.A;  // + k*slot selects chunk k
   for (int i = threadIdx.x; i < KA; i += blockDim.x) {
-    xs[i] = xcol[(i / d.A) * slot + i % d.A];
-    vs[i] = b_out[i % d.A];
+    if (q == 0) xs[i] = xcol[(i / d.A) * slot + i % d.A];
+    vs[i] = 0.f;
   }
   uint32_t phase = 0;
-  for (int w0 = 0; w0 < d.W; w0 += wchunk) {
+  for (int w0 = wbeg; w0 < wbeg + wq; w0 += wchunk) {
     __syncthreads();  // previous chunk consumed
     if (threadIdx.x == 0) {
       // all staging as bulk copies in flight at once: K rows of y_F and the W_out^T slice
@@ -458,6 +463,20 @@ __global__ void __launch_bounds__(kVelThreads)
     }
   }
   __syncthreads();
+  // v = b_out + partials of the cluster's CTAs in rank order, on CTA 0
+  if (nsplit > 1) cluster_sync();  // every partial is complete
+  if (q == 0) {
+    const uint32_t vs_addr = smem_u32(vs);
+    for (int i = threadIdx.x; i < KA; i += blockDim.x) {
+      float v = vs[i];
+      for (int p = 1; p < nsplit; ++p)
+        v += ld_shared_cluster_f32(mapa_shared(vs_addr + 4u * (uint32_t)i, (uint32_t)p));
+      vs[i] = b_out[i % d.A] + v;
+    }
+  }
+  __syncthreads();
+  if (nsplit > 1) cluster_sync();  // the other CTAs may leave once CTA 0 has read them
+  if (q != 0) return;
   const unsigned long long step = *step_idx;
   const float* dtr = dt + (size_t)r * d.K;
   float* colw = buffer + ((size_t)r * d.K * d.H + j) * d.A;
@@ -478,12 +497,16 @@ __global__ void __launch_bounds__(kVelThreads)
   }
 }
 
-// Largest W-chunk (a divisor of W, multiple of 4) whose staging fits ~200 KB.
-// Every bulk copy then starts 16-byte aligned (W and the chunk are multiples of 4).
+// CTAs per velocity cluster: each takes W / nsplit of the width (a multiple of 4).
+static int vel_split(const StepDims& d) { return d.W % 16 == 0 ? 4 : 1; }
+
+// Largest chunk of a CTA's width range (a divisor of it, multiple of 4) whose
+// staging fits ~200 KB.  Every bulk copy then starts 16-byte aligned.
 static int vel_chunk(const StepDims& d) {
   const size_t budget = 200 * 1024 - sizeof(float) * 18 * d.K * d.A;
-  int c = d.W;
-  while (c > 4 && (sizeof(float) * (size_t)(d.K + d.A) * c > budget || d.W % c || c % 4)) --c;
+  const int wq = d.W / vel_split(d);
+  int c = wq;
+  while (c > 4 && (sizeof(float) * (size_t)(d.K + d.A) * c > budget || wq % c || c % 4)) --c;
   return c;
 }
 
@@ -507,9 +530,10 @@ void launch_velocity_euler(const StepDims& d, const float* yF, const float* w_ou
                            const float* b_out, const float* dt, float* buffer, float* out_chunk,
                            float* vel_out, const float* fresh, unsigned long long seed,
                            const unsigned long long* step_idx, cudaStream_t s) {
-  launch_pdl(velocity_euler_kernel, dim3(d.H, d.B), dim3(kVelThreads), vel_smem_bytes(d), s, d,
-             yF, w_out_t, b_out, dt, buffer, out_chunk, vel_out, fresh, seed, step_idx,
-             vel_chunk(d));
+  const int ns = vel_split(d);
+  launch_pdl_cluster(velocity_euler_kernel, dim3(ns, d.H, d.B), dim3(kVelThreads),
+                     vel_smem_bytes(d), s, ns, d, yF, w_out_t, b_out, dt, buffer, out_chunk,
+                     vel_out, fresh, seed, step_idx, vel_chunk(d), ns);
 }
 
 // ----------------------------------------------------------------------------
