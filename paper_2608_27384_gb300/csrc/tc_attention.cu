@@ -342,6 +342,14 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
   const int nsplit = (nkb_tile + kBlocksPerSplit - 1) / kBlocksPerSplit;
   if (nsplit <= 1 || nsplit > a.max_splits) return;  // written by the attention kernel / bad size
   const size_t tbase = (size_t)(r * a.tiles_per_req + gtile) * a.max_splits;
+  // the first 8 splits' partial rows are requested together with the (max, sum)
+  // pairs, so both round trips overlap
+  uint4 x[8];
+#pragma unroll
+  for (int u = 0; u < 8; ++u)
+    if (u < nsplit)
+      x[u] = __ldcg(reinterpret_cast<const uint4*>(
+          (const bf16*)a.part_o + ((tbase + u) * kRows + row) * kDH + lane * 8));
   float2 ml = make_float2(-INFINITY, 0.f);
   if (lane < nsplit) ml = __ldcg(a.part_ml + (tbase + lane) * kRows + row);
   float m_all = warp_max(ml.y > 0.f ? ml.x : -INFINITY);
@@ -351,12 +359,11 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
   const float inv = tot > 0.f ? 1.f / tot : 0.f;  // no visible key in any split: zeros
   float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
   for (int s0 = 0; s0 < nsplit; s0 += 8) {  // up to 8 splits' loads in flight
-    uint4 x[8];
     float ws[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       ws[u] = __shfl_sync(0xffffffffu, w, (s0 + u) & 31);
-      if (s0 + u < nsplit)
+      if (s0 > 0 && s0 + u < nsplit)
         x[u] = __ldcg(reinterpret_cast<const uint4*>(
             (const bf16*)a.part_o + ((tbase + s0 + u) * kRows + row) * kDH + lane * 8));
     }
