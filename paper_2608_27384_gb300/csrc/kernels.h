@@ -117,7 +117,7 @@ constexpr int kBnQKV = 128;
 constexpr int kBnGU = 256;
 constexpr int kBnResid = 128;
 constexpr int kBnTime = 64;
-constexpr int kBnFilm = 256;
+constexpr int kBnFilm = 128;
 
 // Prepare kernel attributes (max dynamic shared memory); call once per device.
 cudaError_t tc_gemm_init();

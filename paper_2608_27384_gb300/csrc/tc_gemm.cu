@@ -35,6 +35,9 @@ struct GemmCfg {
   static constexpr int kStages = (BN <= 64) ? 8 : (BN <= 128 ? 6 : 4);
   static constexpr int kTmemCols = BN < 32 ? 32 : BN;
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/;
+  // full[kStages], empty[kStages], acc_full and the TMEM slot fit the 256-byte area
+  static_assert((2 * kStages + 1) * 8 + 4 <= 256, "barrier area too small for the ring");
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory above the per-CTA limit");
 };
 
 template <int BN, int MODE>
@@ -169,9 +172,14 @@ struct GemmStreamCfg {
   static constexpr int kATx = kABytes;
   static constexpr int kBBytes = BN * kBK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStages = 6;
+  // as many ring stages as fit next to the barriers and the epilogue stages
+  static constexpr int kEpiBytes = 4 * 32 * 144;
+  static constexpr int kStages = (227 * 1024 - 1024 - 256 - kEpiBytes) / kStageBytes;
   // ring + barriers (256 B) + four 32 x 144 B epilogue stages
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256 + 4 * 32 * 144;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256 + kEpiBytes;
+  // full[kStages], empty[kStages], acc_full[2], acc_empty[2], drain and the TMEM slot
+  static_assert((2 * kStages + 5) * 8 + 4 <= 256, "barrier area too small for the ring");
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory above the per-CTA limit");
 };
 
 template <int BN, int MODE>
