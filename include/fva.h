@@ -109,6 +109,9 @@ typedef struct fva_handle fva_handle;
  * post-attention part as one persistent kernel (FVA_K_BLOCK) instead of one
  * launch per operation, where the sizes allow it (width a multiple of 256 up to
  * 1024); results agree within the bf16 tolerances, not bit for bit.
+ * FVA_GEMM_PERSIST=0 (read here) turns off the persistent form of the bf16
+ * projections, which is otherwise used when a projection has at least two output
+ * tiles per SM and no K-split (large batches); both forms give identical results.
  */
 fva_status fva_create(const fva_config* cfg, fva_handle** out);
 

@@ -130,6 +130,7 @@ struct fva_handle {
   int n_sms = 0;
   // fused post-attention block kernel (bf16): task lists per batch size
   bool block_on = false;
+  bool persist_on = true;  // persistent GEMMs where tiles >= 2 x SMs (FVA_GEMM_PERSIST=0: off)
   int blk_split_o = 1, blk_split_d = 1;
   BlockTask* blk_tasks = nullptr;
   std::vector<int> blk_off, blk_n;  // [2 * (B - 1) + last]
@@ -404,6 +405,8 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
     // kernels are faster (every stage of the block kernel still waits for the
     // previous one, and its early weight prefetch competes with epilogue stores
     // for the SM's memory port)
+    const char* penv = std::getenv("FVA_GEMM_PERSIST");
+    h->persist_on = !(penv && penv[0] == '0');
     const char* env = std::getenv("FVA_BLOCK_KERNEL");
     const bool wanted = env && env[0] == '1';
     BlockShape bs{h->Mmax, h->W, h->F, h->Dq, h->N_qkv, h->blk_split_o, h->blk_split_d, true};
@@ -920,6 +923,15 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   const int m_tiles = (M + 127) / 128;
   const int sp_o = bf ? choose_splits(m_tiles * (W / kBnResid), Dq / 64) : 1;
   const int sp_d = bf ? choose_splits(m_tiles * (W / kBnResid), F / 64) : 1;
+  // a projection with at least two tiles per SM and no K-split runs persistent,
+  // so each tile's epilogue overlaps the next tile's MMAs
+  auto gemm = [&](int bn, int mode, const CUtensorMap* ma, const CUtensorMap* mb,
+                  const GemmEpi& e, int Mr, int N, int Kd, int splits) {
+    const long long tiles = (long long)((Mr + 127) / 128) * (N / bn);
+    if (h->persist_on && splits == 1 && h->n_sms > 0 && tiles >= 2LL * h->n_sms)
+      return launch_tc_gemm_persist(bn, mode, ma, mb, e, Mr, N, Kd, h->n_sms, s);
+    return launch_tc_gemm(bn, mode, ma, mb, e, Mr, N, Kd, splits, s);
+  };
   const long long pstride = (long long)M * W;
 
   for (int l = 0; l < L; ++l) {
@@ -948,7 +960,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.nq = h->nq;
       ep.dh = h->dh;
       mark(FVA_K_QKV, l);
-      CUDA_TRY(launch_tc_gemm(kBnQKV, GEMM_QKV_ROPE, &h->m_y, &lw.m_qkv, ep, M, h->N_qkv, W, 1, s));
+      CUDA_TRY(gemm(kBnQKV, GEMM_QKV_ROPE, &h->m_y, &lw.m_qkv, ep, M, h->N_qkv, W, 1));
     } else {
       launch_f32_gemm((float*)h->y, W, (float*)lw.w_qkv, h->c32, h->N_qkv, M, h->N_qkv, W, s);
       launch_f32_qkv_rope(h->c32, (float*)h->q, (float*)kc_l, (float*)vc_l, h->prefix_len_dev,
@@ -1050,7 +1062,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.ldo = W;
       ep.split_stride = pstride;
       mark(FVA_K_OUT_PROJ, l);
-      CUDA_TRY(launch_tc_gemm(kBnResid, GEMM_PARTIAL_BF16, &h->m_attn, &lw.m_o, ep, M, W, Dq, sp_o, s));
+      CUDA_TRY(gemm(kBnResid, GEMM_PARTIAL_BF16, &h->m_attn, &lw.m_o, ep, M, W, Dq, sp_o));
     } else {
       launch_f32_gemm((float*)h->attn, Dq, (float*)lw.w_o, h->part, W, M, W, Dq, s);
     }
@@ -1068,12 +1080,12 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.out = h->mlp;
       ep.ldo = F;
       mark(FVA_K_GATE_UP, l);
-      CUDA_TRY(launch_tc_gemm(kBnGU, GEMM_GEGLU, &h->m_y, &lw.m_gu, ep, M, 2 * F, W, 1, s));
+      CUDA_TRY(gemm(kBnGU, GEMM_GEGLU, &h->m_y, &lw.m_gu, ep, M, 2 * F, W, 1));
       ep.out = h->part;
       ep.ldo = W;
       ep.split_stride = pstride;
       mark(FVA_K_DOWN, l);
-      CUDA_TRY(launch_tc_gemm(kBnResid, GEMM_PARTIAL_BF16, &h->m_mlp, &lw.m_d, ep, M, W, F, sp_d, s));
+      CUDA_TRY(gemm(kBnResid, GEMM_PARTIAL_BF16, &h->m_mlp, &lw.m_d, ep, M, W, F, sp_d));
     } else {
       launch_f32_gemm((float*)h->y, W, (float*)lw.w_gu, h->c32, 2 * F, M, 2 * F, W, s);
       launch_f32_geglu(h->c32, (float*)h->mlp, M, F, s);

@@ -128,6 +128,13 @@ cudaError_t launch_tc_gemm(int bn, int mode, const CUtensorMap* a, const CUtenso
                            const GemmEpi& ep, int M, int N, int K, int splits,
                            cudaStream_t s);
 
+// Persistent form for many tiles: min(grid, tiles) CTAs walk the (row tile,
+// column tile) grid with two TMEM accumulators, no split-K.  bn/mode:
+// (kBnQKV, QKV_ROPE), (kBnGU, GEGLU), (kBnResid, PARTIAL_BF16).
+cudaError_t launch_tc_gemm_persist(int bn, int mode, const CUtensorMap* a, const CUtensorMap* b,
+                                   const GemmEpi& ep, int M, int N, int K, int grid,
+                                   cudaStream_t s);
+
 // Persistent weight-streaming form of (kBnFilm, BIAS_F32) for M <= 128 rows: at
 // most `grid` CTAs (one per SM) walk the N / kBnFilm column tiles.
 cudaError_t launch_tc_gemm_stream(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep,

@@ -310,6 +310,180 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ---------------------------------------------------------------------------
+// Persistent form of the per-op GEMM for shapes with many more tiles than SMs:
+// each CTA walks tiles t = blockIdx.x, + gridDim.x, ... (row tile t % m_tiles,
+// column tile t / m_tiles, so concurrent CTAs share a weight tile) through one
+// continuous load ring, with two TMEM accumulators so that the epilogue of one
+// tile runs under the MMAs of the next.  No split-K.
+// ---------------------------------------------------------------------------
+template <int BN>
+struct GemmPersistCfg {
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kEpiBytes = 4 * 32 * 144;
+  static constexpr int kStages = (227 * 1024 - 1024 - 256 - kEpiBytes) / kStageBytes;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256 + kEpiBytes;
+  // full[kStages], empty[kStages], acc_full[2], acc_empty[2], drain and the TMEM slot
+  static_assert((2 * kStages + 5) * 8 + 4 <= 256, "barrier area too small for the ring");
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory above the per-CTA limit");
+  static_assert(2 * BN <= 512, "two accumulators must fit TMEM");
+};
+
+template <int BN, int MODE>
+__global__ void __launch_bounds__(kThreads, 1)
+    tc_gemm_persist_kernel(const __grid_constant__ CUtensorMap tmA,
+                           const __grid_constant__ CUtensorMap tmB, const GemmEpi ep, int M,
+                           int m_tiles, int n_tiles, int nkb) {
+  using C = GemmPersistCfg<BN>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint64_t* full = (uint64_t*)(smem + C::kStages * C::kStageBytes);
+  uint64_t* empty = full + C::kStages;
+  uint64_t* acc_full = empty + C::kStages;  // [2]
+  uint64_t* acc_empty = acc_full + 2;       // [2]
+  uint64_t* drain = acc_empty + 2;
+  uint32_t* tmem_slot = (uint32_t*)(drain + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tiles = m_tiles * n_tiles;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 4);  // one arrival per epilogue warp
+    }
+    mbar_init(drain, 1);
+    fence_barrier_init();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 2 * BN);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+
+  if (warp == 0 && lane == 0) {
+    // ---------------- TMA producer: the first tile's weight stages go out
+    // before waiting for the predecessor grid, which writes A
+    const int t0 = blockIdx.x;
+    const int pre = t0 < tiles ? min(nkb, C::kStages) : 0;
+    for (int i = 0; i < pre; ++i) {
+      mbar_arrive_expect_tx(&full[i], C::kStageBytes);
+      tma_load_2d(smem + i * C::kStageBytes + C::kABytes, &tmB, i * kBK, (t0 / m_tiles) * BN,
+                  &full[i]);
+    }
+    pdl_wait();
+    for (int i = 0; i < pre; ++i)
+      tma_load_2d(smem + i * C::kStageBytes, &tmA, i * kBK, (t0 % m_tiles) * kBM, &full[i]);
+    uint32_t it = 0;
+    bool ok = true;
+    for (int t = t0; ok && t < tiles; t += gridDim.x) {
+      const int m0 = (t % m_tiles) * kBM, n0 = (t / m_tiles) * BN;
+      for (int i = 0; i < nkb; ++i, ++it) {
+        if (it < (uint32_t)pre) continue;  // issued above
+        const int s = it % C::kStages;
+        if (!mbar_wait(&empty[s], ((it / C::kStages) & 1u) ^ 1u, ep.err, KERR_WAIT_MMA)) {
+          ok = false;
+          break;
+        }
+        uint8_t* sa = smem + s * C::kStageBytes;
+        mbar_arrive_expect_tx(&full[s], C::kStageBytes);
+        tma_load_2d(sa, &tmA, i * kBK, m0, &full[s]);
+        tma_load_2d(sa + C::kABytes, &tmB, i * kBK, n0, &full[s]);
+      }
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---------------- MMA issuer
+    constexpr uint32_t idesc = umma_idesc_bf16(kBM, BN, false);
+    uint32_t it = 0, acc = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; ok && t < tiles; t += gridDim.x, ++acc) {
+      const uint32_t buf = acc & 1u;
+      if (!mbar_wait(&acc_empty[buf], ((acc >> 1) & 1u) ^ 1u, ep.err, KERR_WAIT_SYNC)) break;
+      tc_fence_after();
+      const uint32_t d = tmem + buf * BN;
+      for (int i = 0; i < nkb; ++i, ++it) {
+        const int s = it % C::kStages;
+        if (!mbar_wait(&full[s], (it / C::kStages) & 1u, ep.err, KERR_WAIT_TMA)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t sa = smem_u32(smem + s * C::kStageBytes);
+        const uint32_t sb = sa + C::kABytes;
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk) {
+          const uint64_t ad = umma_desc_sw128(sa + kk * 32, 16, 1024);
+          const uint64_t bd = umma_desc_sw128(sb + kk * 32, 16, 1024);
+          umma_bf16(d, ad, bd, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+        }
+        umma_commit(&empty[s]);
+      }
+      if (ok) umma_commit(&acc_full[buf]);
+    }
+    // every MMA of this thread completes before TMEM is released
+    umma_commit(drain);
+    mbar_wait(drain, 0, nullptr, 0);
+  } else if (warp >= 2) {
+    // ---------------- epilogue: one output row per thread
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    uint8_t* stage = smem + C::kStages * C::kStageBytes + 256 + (warp - 2) * (32 * 144);
+    uint32_t acc = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++acc) {
+      const int m0 = (t % m_tiles) * kBM, n0 = (t / m_tiles) * BN;
+      const uint32_t buf = acc & 1u;
+      uint4 rh[MODE == GEMM_QKV_ROPE ? BN / 8 : 1];
+      if constexpr (MODE == GEMM_QKV_ROPE) gemm_epilogue_load_rope<BN>(ep, m0 + row, M, n0, rh);
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&acc_full[buf], (acc >> 1) & 1u, ep.err,
+                                                     KERR_WAIT_MMA));
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t trow = tmem + buf * BN + ((uint32_t)(quarter * 32) << 16);
+      if constexpr (MODE == GEMM_QKV_ROPE)
+        gemm_epilogue_qkv<BN>(ep, trow, m0 + row, M, n0, stage, lane, rh);
+      else
+        gemm_epilogue<BN, MODE>(ep, trow, m0 + row, M, n0, 0, stage, lane);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[buf]);
+    }
+  }
+  // the producer and MMA lanes rejoin their warps first: a CTA barrier reached
+  // by a split warp does not wait for the rest of the CTA
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 2 * BN);
+  }
+}
+
+template <int BN, int MODE>
+cudaError_t set_attr_persist() {
+  return cudaFuncSetAttribute(tc_gemm_persist_kernel<BN, MODE>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              GemmPersistCfg<BN>::kSmemBytes);
+}
+
+template <int BN, int MODE>
+cudaError_t launch_persist(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep, int M,
+                           int N, int K, int grid, cudaStream_t s) {
+  const int m_tiles = (M + kBM - 1) / kBM, n_tiles = N / BN;
+  return launch_pdl(tc_gemm_persist_kernel<BN, MODE>, dim3(std::min(grid, m_tiles * n_tiles)),
+                    dim3(kThreads), GemmPersistCfg<BN>::kSmemBytes, s, *a, *b, ep, M, m_tiles,
+                    n_tiles, K / kBK);
+}
+
 template <int BN, int MODE>
 cudaError_t set_attr() {
   return cudaFuncSetAttribute(tc_gemm_kernel<BN, MODE>,
@@ -341,7 +515,24 @@ cudaError_t tc_gemm_init() {
   if ((e = set_attr<kBnResid, GEMM_PARTIAL_F32>()) != cudaSuccess) return e;
   if ((e = set_attr<kBnResid, GEMM_PARTIAL_BF16>()) != cudaSuccess) return e;
   if ((e = set_attr<kBnGU, GEMM_GEGLU>()) != cudaSuccess) return e;
+  if ((e = set_attr_persist<kBnQKV, GEMM_QKV_ROPE>()) != cudaSuccess) return e;
+  if ((e = set_attr_persist<kBnGU, GEMM_GEGLU>()) != cudaSuccess) return e;
+  if ((e = set_attr_persist<kBnResid, GEMM_PARTIAL_BF16>()) != cudaSuccess) return e;
   return cudaSuccess;
+}
+
+cudaError_t launch_tc_gemm_persist(int bn, int mode, const CUtensorMap* a, const CUtensorMap* b,
+                                   const GemmEpi& ep, int M, int N, int K, int grid,
+                                   cudaStream_t s) {
+  if (M <= 0) return cudaSuccess;
+  if (N % bn != 0 || K % kBK != 0 || grid < 1) return cudaErrorInvalidValue;
+  if (bn == kBnQKV && mode == GEMM_QKV_ROPE)
+    return launch_persist<kBnQKV, GEMM_QKV_ROPE>(a, b, ep, M, N, K, grid, s);
+  if (bn == kBnGU && mode == GEMM_GEGLU)
+    return launch_persist<kBnGU, GEMM_GEGLU>(a, b, ep, M, N, K, grid, s);
+  if (bn == kBnResid && mode == GEMM_PARTIAL_BF16)
+    return launch_persist<kBnResid, GEMM_PARTIAL_BF16>(a, b, ep, M, N, K, grid, s);
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_tc_gemm(int bn, int mode, const CUtensorMap* a, const CUtensorMap* b,

@@ -347,3 +347,24 @@ def test_step_profile_matches_step_and_counts_launches():
         assert all(us > 0 for _, _, us in recs)
     finally:
         case.close()
+
+
+def test_persistent_gemm_bitwise(monkeypatch):
+    """The persistent projections (used where a projection has at least two
+    output tiles per SM) give the per-operation kernels' results bit for bit:
+    the same MMAs in the same order per tile, the same epilogues.  128 requests
+    of 160 tokens make every projection of this reduced expert persistent."""
+    wl = WL.small_bf16_workload(batch=128, n_chunks=4, chunk_tokens=40, prefix_lens=[64] * 128)
+    fresh = WL.make_fresh_noise(wl, 1)[0]
+    results = {}
+    for mode in ("1", "0"):
+        monkeypatch.setenv("FVA_GEMM_PERSIST", mode)
+        case = Case(wl)
+        try:
+            results[mode] = case.run(fresh=fresh)
+        finally:
+            case.close()
+    for key in ("out", "buffer", "vel"):
+        a, b = results["1"][key], results["0"][key]
+        assert np.isfinite(a).all()
+        assert np.array_equal(a.view(np.uint32), b.view(np.uint32)), key
