@@ -294,11 +294,92 @@ __global__ void resid_norm_kernel(StepDims d, float* __restrict__ h,
                           y + (size_t)m * d.W);
 }
 
+// The same operation for many rows: R rows per CTA (W = 4 x blockDim, at most
+// two partial planes), every row's loads in flight before any reduction, one
+// shared-memory exchange for the R row sums.  With one row per CTA the register
+// budget keeps four rows per SM in flight, too few to cover DRAM latency when
+// the activations no longer fit L2.
+template <typename Act, typename Part, int R>
+__global__ void __launch_bounds__(256)
+    resid_norm_rows_kernel(StepDims d, int rows, float* __restrict__ h,
+                           const Part* __restrict__ part, int n_parts, long long part_stride,
+                           const float* __restrict__ mod, int gate_off, int scale_off,
+                           int shift_off, Act* __restrict__ y) {
+  __shared__ float red[R][8];
+  const int m0 = blockIdx.x * R;
+  const int col = threadIdx.x * 4;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  pdl_trigger();
+  pdl_wait();
+  float4 hv[R], acc[R], g[R], sc[R], sh[R];
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    const int m = min(m0 + r, rows - 1);  // rows past the end repeat the last (not stored)
+    const int rq = m / d.T, c = (m % d.T) / d.H;
+    const float* mrow = mod + (size_t)(rq * d.K + c) * d.N_mod;
+    acc[r] = load4_cg(part + (size_t)m * d.W + col);
+    if (n_parts > 1) {
+      const float4 q = load4_cg(part + part_stride + (size_t)m * d.W + col);
+      acc[r].x += q.x; acc[r].y += q.y; acc[r].z += q.z; acc[r].w += q.w;
+    }
+    hv[r] = *reinterpret_cast<const float4*>(h + (size_t)m * d.W + col);
+    g[r] = *reinterpret_cast<const float4*>(mrow + gate_off + col);
+    sc[r] = *reinterpret_cast<const float4*>(mrow + scale_off + col);
+    sh[r] = *reinterpret_cast<const float4*>(mrow + shift_off + col);
+  }
+  float ss[R];
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    hv[r].x = fmaf(g[r].x, acc[r].x, hv[r].x);
+    hv[r].y = fmaf(g[r].y, acc[r].y, hv[r].y);
+    hv[r].z = fmaf(g[r].z, acc[r].z, hv[r].z);
+    hv[r].w = fmaf(g[r].w, acc[r].w, hv[r].w);
+    if (m0 + r < rows) *reinterpret_cast<float4*>(h + (size_t)(m0 + r) * d.W + col) = hv[r];
+    ss[r] = warp_sum(hv[r].x * hv[r].x + hv[r].y * hv[r].y + hv[r].z * hv[r].z +
+                     hv[r].w * hv[r].w);
+    if (lane == 0) red[r][warp] = ss[r];
+  }
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) t += red[r][w];
+    const float rn = rsqrtf(t / (float)d.W + d.eps);
+    if (m0 + r < rows)
+      store4<Act>(y + (size_t)(m0 + r) * d.W + col, hv[r].x * rn * (1.f + sc[r].x) + sh[r].x,
+                  hv[r].y * rn * (1.f + sc[r].y) + sh[r].y,
+                  hv[r].z * rn * (1.f + sc[r].z) + sh[r].z,
+                  hv[r].w * rn * (1.f + sc[r].w) + sh[r].w);
+  }
+}
+
+static int device_sms() {
+  static int n = [] {
+    int dev = 0, v = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+    return v > 0 ? v : 1;
+  }();
+  return n;
+}
+
 template <typename Part>
 static void launch_resid_norm_t(const StepDims& d, int rows, float* h, const Part* part,
                                 int n_parts, long long part_stride, const float* mod,
                                 int gate_off, int scale_off, int shift_off, void* y,
                                 bool act_bf16, cudaStream_t s) {
+  constexpr int R = 4;
+  if (d.W == 1024 && n_parts <= 2 && rows >= R * 4 * device_sms()) {
+    const dim3 grid((rows + R - 1) / R);
+    if (act_bf16)
+      launch_pdl(resid_norm_rows_kernel<bf16, Part, R>, grid, dim3(256), 0, s, d, rows, h, part,
+                 n_parts, part_stride, mod, gate_off, scale_off, shift_off, (bf16*)y);
+    else
+      launch_pdl(resid_norm_rows_kernel<float, Part, R>, grid, dim3(256), 0, s, d, rows, h, part,
+                 n_parts, part_stride, mod, gate_off, scale_off, shift_off, (float*)y);
+    return;
+  }
   if (act_bf16)
     launch_pdl(resid_norm_kernel<bf16, Part>, dim3(rows), dim3(row_threads(d.W)), 0, s, d, h,
                part, n_parts, part_stride, mod, gate_off, scale_off, shift_off, (bf16*)y);
