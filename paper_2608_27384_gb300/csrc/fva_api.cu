@@ -875,6 +875,15 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   // ---- per-chunk FiLM condition and modulation (App. A.4)
   mark(FVA_K_TIMESTEP_EMBED, -1);
   launch_temb(h->tau_dev(), h->temb_freq, BK, W, h->temb, bf, s);
+  // a projection with at least two tiles per SM and no K-split runs persistent,
+  // so each tile's epilogue overlaps the next tile's MMAs
+  auto gemm = [&](int bn, int mode, const CUtensorMap* ma, const CUtensorMap* mb,
+                  const GemmEpi& e, int Mr, int N, int Kd, int splits) {
+    const long long tiles = (long long)((Mr + 127) / 128) * (N / bn);
+    if (h->persist_on && splits == 1 && h->n_sms > 0 && tiles >= 2LL * h->n_sms)
+      return launch_tc_gemm_persist(bn, mode, ma, mb, e, Mr, N, Kd, h->n_sms, s);
+    return launch_tc_gemm(bn, mode, ma, mb, e, Mr, N, Kd, splits, s);
+  };
   GemmEpi ep{};
   ep.err = h->err_dev;
   if (bf) {
@@ -904,8 +913,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     mark(FVA_K_FILM, -1);
     CUDA_TRY(BK <= 16 ? launch_tc_gemm_stream(&h->m_cond16, &h->m_wmod, ep, BK, h->N_mod, W,
                                               h->n_sms, s)
-                       : launch_tc_gemm(kBnFilm, GEMM_BIAS_F32, &h->m_cond, &h->m_wmod, ep, BK,
-                                        h->N_mod, W, 1, s));
+                       : gemm(kBnFilm, GEMM_BIAS_F32, &h->m_cond, &h->m_wmod, ep, BK, h->N_mod, W, 1));
   } else {
     launch_f32_gemm((float*)h->temb, W, (float*)h->w_t1, h->c32, W, BK, W, W, s);
     launch_f32_bias_act(h->c32, h->b_t1, (float*)h->t1, BK, W, true, s);
@@ -923,15 +931,6 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   const int m_tiles = (M + 127) / 128;
   const int sp_o = bf ? choose_splits(m_tiles * (W / kBnResid), Dq / 64) : 1;
   const int sp_d = bf ? choose_splits(m_tiles * (W / kBnResid), F / 64) : 1;
-  // a projection with at least two tiles per SM and no K-split runs persistent,
-  // so each tile's epilogue overlaps the next tile's MMAs
-  auto gemm = [&](int bn, int mode, const CUtensorMap* ma, const CUtensorMap* mb,
-                  const GemmEpi& e, int Mr, int N, int Kd, int splits) {
-    const long long tiles = (long long)((Mr + 127) / 128) * (N / bn);
-    if (h->persist_on && splits == 1 && h->n_sms > 0 && tiles >= 2LL * h->n_sms)
-      return launch_tc_gemm_persist(bn, mode, ma, mb, e, Mr, N, Kd, h->n_sms, s);
-    return launch_tc_gemm(bn, mode, ma, mb, e, Mr, N, Kd, splits, s);
-  };
   const long long pstride = (long long)M * W;
 
   for (int l = 0; l < L; ++l) {

@@ -15,11 +15,13 @@
 //   warp 1      TMEM (512 columns: S in 0..255, O in 256..511); one lane issues
 //               S = Q K^T as one MMA per 16 head dims with N = all the split's
 //               keys (each Q and K byte is read from shared memory once), and,
-//               after the softmax, O = P V (M=128, N=256, MN-major V);
-//   warps 2..17 softmax + epilogue, four threads per query row (one per
-//               64-key block / 64 head-dim columns): block max, row max through
-//               shared memory, P = exp(S - row max) as bf16 over the Q tile (Q is
-//               dead once S is complete) with the row's sum; then O from TMEM.
+//               per key block, once its P is written, O += P V (M=128, N=256,
+//               A = P from TMEM, MN-major V from shared memory);
+//   warps 2..17 softmax + epilogue, four threads per query row (16 keys of every
+//               block / 64 head-dim columns): block max, row max through shared
+//               memory, P = exp(S - row max) as bf16 pairs written back over S's
+//               TMEM columns (S is dead once every thread holds its values), with
+//               the row's sum; then O from TMEM.
 // K and V live slab-major: head-dim slab j (64 values, 128 bytes) of key k is
 // at j * 32 KB + k * 128 bytes, so the split's keys form one uniformly strided
 // operand for the S MMA and V's head-dim slabs are 32 KB apart for the P V MMA.
@@ -70,7 +72,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-  uint8_t* sQP = smem;                      // 4 slabs [128 rows x 128 B]: Q, then P
+  uint8_t* sQP = smem;                      // 4 slabs [128 rows x 128 B]: Q
   uint8_t* sKV = smem + kQBytes;            // 4 slabs [256 keys x 128 B]: K, then V
   uint64_t* bars = (uint64_t*)(sKV + kBlocksPerSplit * kKVBytes);
   uint64_t* qk_full = bars + 0;   // [4]: head-dim slab j of Q and of every K block
@@ -175,11 +177,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
 #pragma unroll
       for (int ks = 0; ks < kKB / 16; ++ks) {
-        const uint64_t ad = umma_desc_sw128(qp_base + j * (kRows * 128) + ks * 32, 16, 1024);
-        // V keys j*64 + 16 ks .. +15, all 256 head dims: MN-major B operand whose
-        // 64-wide head-dim slabs are kSlabK apart.
+        // P keys j*64 + 16 ks .. +15 from TMEM (bf16 pairs, 8 columns); V the same
+        // keys, all 256 head dims: MN-major B operand whose 64-wide head-dim slabs
+        // are kSlabK apart.
         const uint64_t bd = umma_desc_sw128(kv_base + (j * kKB + ks * 16) * 128, kSlabK, 1024);
-        umma_bf16(tO, ad, bd, idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
+        umma_bf16_ts(tO, tS + j * (kKB / 2) + ks * 8, bd, idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
       }
     }
     if (good) umma_commit(o_full);
@@ -231,8 +233,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     xmax[g * kRows + row] = mx;
-    // S is complete (every thread waited for its commit), so past this barrier Q
-    // is dead for all threads and P may go over it
+    // every thread holds its S values past this barrier, so P may go over S's
+    // TMEM columns
     softmax_bar();
     float mrow = xmax[row];
 #pragma unroll
@@ -244,7 +246,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (j >= nblk) break;
       if (good) {
         // P = exp(S - row max) over visible keys, rounded to bf16 (the row sum
-        // adds the rounded values the P V MMA uses), 128-byte swizzled over Q
+        // adds the rounded values the P V MMA uses)
         const bool all_vis = block_all_vis(j);
         uint32_t w[8];
 #pragma unroll
@@ -260,13 +262,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           l2[0] += __uint_as_float(w[i / 2] << 16);
           l2[1] += __uint_as_float(w[i / 2] & 0xFFFF0000u);
         }
-        uint8_t* prow = sQP + j * (kRows * 128) + row * 128;
-        *reinterpret_cast<uint4*>(prow + (((2 * g) ^ (row & 7)) * 16)) =
-            make_uint4(w[0], w[1], w[2], w[3]);
-        *reinterpret_cast<uint4*>(prow + (((2 * g + 1) ^ (row & 7)) * 16)) =
-            make_uint4(w[4], w[5], w[6], w[7]);
+        // P of keys j*64 + 16g .. +15 over S's (already read) TMEM columns, as
+        // the A operand of the P V MMAs
+        tmem_st8(tS + lane_off + j * (kKB / 2) + g * 8, w);
+        tmem_st_wait();
       }
-      fence_proxy_async_smem();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_full[j]);
     }
@@ -289,7 +290,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld32_nowait(tO + lane_off + c0, o0);
       tmem_ld32_nowait(tO + lane_off + c0 + 32, o1);
       tmem_ld_wait();
-      // P, Q and K/V are dead once O is complete: each warp stages its 32 rows
+      // Q and K/V are dead once O is complete: each warp stages its 32 rows
       // there for coalesced stores
       uint8_t* stage = smem + (warp - 2) * (32 * 144);
       // one split: the output row; several: this split's partial (O / l, with

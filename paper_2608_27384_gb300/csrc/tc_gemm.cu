@@ -518,6 +518,7 @@ cudaError_t tc_gemm_init() {
   if ((e = set_attr_persist<kBnQKV, GEMM_QKV_ROPE>()) != cudaSuccess) return e;
   if ((e = set_attr_persist<kBnGU, GEMM_GEGLU>()) != cudaSuccess) return e;
   if ((e = set_attr_persist<kBnResid, GEMM_PARTIAL_BF16>()) != cudaSuccess) return e;
+  if ((e = set_attr_persist<kBnFilm, GEMM_BIAS_F32>()) != cudaSuccess) return e;
   return cudaSuccess;
 }
 
@@ -532,6 +533,8 @@ cudaError_t launch_tc_gemm_persist(int bn, int mode, const CUtensorMap* a, const
     return launch_persist<kBnGU, GEMM_GEGLU>(a, b, ep, M, N, K, grid, s);
   if (bn == kBnResid && mode == GEMM_PARTIAL_BF16)
     return launch_persist<kBnResid, GEMM_PARTIAL_BF16>(a, b, ep, M, N, K, grid, s);
+  if (bn == kBnFilm && mode == GEMM_BIAS_F32)
+    return launch_persist<kBnFilm, GEMM_BIAS_F32>(a, b, ep, M, N, K, grid, s);
   return cudaErrorInvalidValue;
 }
 
