@@ -130,6 +130,7 @@ struct fva_handle {
   int n_sms = 0;
   // fused post-attention block kernel (bf16): task lists per batch size
   bool block_on = false;
+  int bn_qkv = kBnQKV, bn_gu = kBnGU;  // tile widths of the QKV and gate/up weight layouts
   bool persist_on = true;  // persistent GEMMs where tiles >= 2 x SMs (FVA_GEMM_PERSIST=0: off)
   int blk_split_o = 1, blk_split_d = 1;
   BlockTask* blk_tasks = nullptr;
@@ -401,16 +402,21 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
     };
     h->blk_split_o = pick(h->Dq / 64, 0);
     h->blk_split_d = pick(h->F / 64, h->F);
+    if (h->Mmax <= 128) {  // one row tile: narrower QKV and gate/up tiles
+      h->bn_qkv = kBnSmall;
+      h->bn_gu = kBnSmall;
+    }
+    const char* penv = std::getenv("FVA_GEMM_PERSIST");
+    h->persist_on = !(penv && penv[0] == '0');
     // opt-in (FVA_BLOCK_KERNEL=1): on the 500-token workloads the per-operation
     // kernels are faster (every stage of the block kernel still waits for the
     // previous one, and its early weight prefetch competes with epilogue stores
     // for the SM's memory port)
-    const char* penv = std::getenv("FVA_GEMM_PERSIST");
-    h->persist_on = !(penv && penv[0] == '0');
     const char* env = std::getenv("FVA_BLOCK_KERNEL");
     const bool wanted = env && env[0] == '1';
     BlockShape bs{h->Mmax, h->W, h->F, h->Dq, h->N_qkv, h->blk_split_o, h->blk_split_d, true};
-    h->block_on = wanted && h->n_sms > 0 && block_supported(bs);
+    h->block_on = wanted && h->n_sms > 0 && h->bn_gu == kBnGU && h->bn_qkv == kBnQKV &&
+                  block_supported(bs);
     if (h->block_on) {
       std::vector<BlockTask> all;
       h->blk_off.assign(2 * h->Bmax, 0);
@@ -667,9 +673,10 @@ extern "C" fva_status fva_load_weights(fva_handle* h, const void* const* tensors
     };
     for (int n2 = 0; n2 < h->N_qkv; ++n2) {
       int src = n2;
-      if (h->bf16) {  // rotate-half partners side by side inside each kBnQKV tile
-        const int half = kBnQKV / 2, seg = n2 / dh, within = n2 % dh;
-        const int tj = within / kBnQKV, c = within % kBnQKV;
+      if (h->bf16) {  // rotate-half partners side by side inside each QKV tile
+        const int bq = h->bn_qkv;
+        const int half = bq / 2, seg = n2 / dh, within = n2 % dh;
+        const int tj = within / bq, c = within % bq;
         const int d = c < half ? tj * half + c : tj * half + (c - half) + dh / 2;
         src = seg * dh + d;
       }
@@ -677,8 +684,9 @@ extern "C" fva_status fva_load_weights(fva_handle* h, const void* const* tensors
     }
     for (int n2 = 0; n2 < 2 * F; ++n2) {
       const float* s;
-      if (h->bf16) {  // gate rows then matching up rows inside each kBnGU tile
-        const int half = kBnGU / 2, j = n2 / kBnGU, c = n2 % kBnGU;
+      if (h->bf16) {  // gate rows then matching up rows inside each gate/up tile
+        const int bg = h->bn_gu;
+        const int half = bg / 2, j = n2 / bg, c = n2 % bg;
         const int f = j * half + (c < half ? c : c - half);
         s = (c < half ? li(l, 8) : li(l, 9)).data() + (size_t)f * W;
       } else {
@@ -733,9 +741,9 @@ extern "C" fva_status fva_load_weights(fva_handle* h, const void* const* tensors
     lw.w_d = base + o_d[l];
     if (h->bf16) {
       fva_status st;
-      if ((st = make_map(&lw.m_qkv, lw.w_qkv, h->N_qkv, W, kBnQKV)) ||
+      if ((st = make_map(&lw.m_qkv, lw.w_qkv, h->N_qkv, W, h->bn_qkv)) ||
           (st = make_map(&lw.m_o, lw.w_o, W, Dq, kBnResid)) ||
-          (st = make_map(&lw.m_gu, lw.w_gu, 2 * F, W, kBnGU)) ||
+          (st = make_map(&lw.m_gu, lw.w_gu, 2 * F, W, h->bn_gu)) ||
           (st = make_map(&lw.m_d, lw.w_d, W, F, kBnResid)))
         return st;
     }
@@ -959,7 +967,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.nq = h->nq;
       ep.dh = h->dh;
       mark(FVA_K_QKV, l);
-      CUDA_TRY(gemm(kBnQKV, GEMM_QKV_ROPE, &h->m_y, &lw.m_qkv, ep, M, h->N_qkv, W, 1));
+      CUDA_TRY(gemm(h->bn_qkv, GEMM_QKV_ROPE, &h->m_y, &lw.m_qkv, ep, M, h->N_qkv, W, 1));
     } else {
       launch_f32_gemm((float*)h->y, W, (float*)lw.w_qkv, h->c32, h->N_qkv, M, h->N_qkv, W, s);
       launch_f32_qkv_rope(h->c32, (float*)h->q, (float*)kc_l, (float*)vc_l, h->prefix_len_dev,
@@ -1079,7 +1087,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.out = h->mlp;
       ep.ldo = F;
       mark(FVA_K_GATE_UP, l);
-      CUDA_TRY(gemm(kBnGU, GEMM_GEGLU, &h->m_y, &lw.m_gu, ep, M, 2 * F, W, 1));
+      CUDA_TRY(gemm(h->bn_gu, GEMM_GEGLU, &h->m_y, &lw.m_gu, ep, M, 2 * F, W, 1));
       ep.out = h->part;
       ep.ldo = W;
       ep.split_stride = pstride;

@@ -115,6 +115,9 @@ struct GemmEpi {
 // Tile widths used for each GEMM of the step (the weight layouts depend on them).
 constexpr int kBnQKV = 128;
 constexpr int kBnGU = 256;
+// QKV and gate/up tile width when every row fits one row tile (B*K*H <= 128):
+// with so few rows the wide tiles leave most SMs idle.
+constexpr int kBnSmall = 64;
 constexpr int kBnResid = 128;
 constexpr int kBnTime = 64;
 constexpr int kBnFilm = 128;

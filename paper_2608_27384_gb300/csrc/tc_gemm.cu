@@ -515,6 +515,8 @@ cudaError_t tc_gemm_init() {
   if ((e = set_attr<kBnResid, GEMM_PARTIAL_F32>()) != cudaSuccess) return e;
   if ((e = set_attr<kBnResid, GEMM_PARTIAL_BF16>()) != cudaSuccess) return e;
   if ((e = set_attr<kBnGU, GEMM_GEGLU>()) != cudaSuccess) return e;
+  if ((e = set_attr<kBnSmall, GEMM_QKV_ROPE>()) != cudaSuccess) return e;
+  if ((e = set_attr<kBnSmall, GEMM_GEGLU>()) != cudaSuccess) return e;
   if ((e = set_attr_persist<kBnQKV, GEMM_QKV_ROPE>()) != cudaSuccess) return e;
   if ((e = set_attr_persist<kBnGU, GEMM_GEGLU>()) != cudaSuccess) return e;
   if ((e = set_attr_persist<kBnResid, GEMM_PARTIAL_BF16>()) != cudaSuccess) return e;
@@ -554,6 +556,10 @@ cudaError_t launch_tc_gemm(int bn, int mode, const CUtensorMap* a, const CUtenso
     return launch<kBnResid, GEMM_PARTIAL_BF16>(a, b, ep, M, N, K, splits, s);
   if (bn == kBnGU && mode == GEMM_GEGLU)
     return launch<kBnGU, GEMM_GEGLU>(a, b, ep, M, N, K, splits, s);
+  if (bn == kBnSmall && mode == GEMM_QKV_ROPE)
+    return launch<kBnSmall, GEMM_QKV_ROPE>(a, b, ep, M, N, K, splits, s);
+  if (bn == kBnSmall && mode == GEMM_GEGLU)
+    return launch<kBnSmall, GEMM_GEGLU>(a, b, ep, M, N, K, splits, s);
   return cudaErrorInvalidValue;
 }
 
