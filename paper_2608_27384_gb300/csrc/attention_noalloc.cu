@@ -128,6 +128,7 @@ extern "C" fva_status fva_chunk_attention_noalloc(const void* q, const void* k, 
   a.nq = n_q_heads;
   a.S_cap = kv_rows;
   a.tiles_per_req = (int)tiles;
+  a.blocks_per_split = kAttnKeysPerSplit / kAttnKeyBlock;
   a.max_splits = (int)splits;
   a.kv_row0 = 0;
   a.scale_log2 = 1.4426950408889634f / 16.0f;  // log2(e) / sqrt(256)

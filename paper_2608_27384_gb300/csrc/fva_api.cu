@@ -126,7 +126,7 @@ struct fva_handle {
   bool bf16 = true;
   size_t act = 2;  // bytes per activation / weight element
   int W, nq, dh, Dq, F, A, K, H, T, L, Bmax, Pmax, S_cap, N_qkv, N_mod, BKmax, Mmax;
-  int tiles_per_req = 0, attn_max_splits = 0;
+  int tiles_per_req = 0, attn_max_splits = 0, attn_bps = 4;
   int n_sms = 0;
   // fused post-attention block kernel (bf16): task lists per batch size
   bool block_on = false;
@@ -451,7 +451,16 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
   }
   if (h->bf16) {
     h->tiles_per_req = (h->T * h->nq + 127) / 128;
-    h->attn_max_splits = (h->S_cap + kAttnKeysPerSplit - 1) / kAttnKeysPerSplit;
+    // 64-key blocks per split: the largest of 4, 2, 1 that still gives about half
+    // as many CTAs as SMs (few query tiles: short splits), at most 32 splits
+    const int nkb_max = (h->S_cap + 63) / 64;
+    h->attn_bps = 4;
+    while (h->attn_bps > 1 &&
+           (long long)h->tiles_per_req * h->Bmax * ((nkb_max + h->attn_bps - 1) / h->attn_bps) <
+               std::max(1, h->n_sms / 2))
+      h->attn_bps /= 2;
+    while ((nkb_max + h->attn_bps - 1) / h->attn_bps > 32 && h->attn_bps < 4) h->attn_bps *= 2;
+    h->attn_max_splits = (nkb_max + h->attn_bps - 1) / h->attn_bps;
     const size_t tiles = (size_t)h->Bmax * h->tiles_per_req;
     if ((st = dalloc(h, &h->att_part_o, tiles * h->attn_max_splits * 128 * 256)) ||
         (st = dalloc(h, &h->att_part_ml, tiles * h->attn_max_splits * 128)))
@@ -991,6 +1000,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       aa.S_cap = h->S_cap;
       aa.tiles_per_req = h->tiles_per_req;
       aa.max_splits = h->attn_max_splits;
+      aa.blocks_per_split = h->attn_bps;
       aa.kv_row0 = l * h->Bmax * h->S_cap;
       aa.scale_log2 = 1.4426950408889634f / std::sqrt((float)h->dh);
       aa.err = h->err_dev;
@@ -1401,6 +1411,7 @@ extern "C" fva_status fva_chunk_attention(fva_handle* h, const void* q, const vo
   aa.S_cap = kv_rows;
   aa.tiles_per_req = h->tiles_per_req;
   aa.max_splits = (kv_rows + kAttnKeysPerSplit - 1) / kAttnKeysPerSplit;
+  aa.blocks_per_split = kAttnKeysPerSplit / kAttnKeyBlock;
   aa.kv_row0 = 0;
   aa.scale_log2 = 1.4426950408889634f / std::sqrt((float)h->dh);
   aa.err = h->err_dev;

@@ -150,6 +150,7 @@ struct AttnArgs {
   void* part_o;         // bf16 [B*tiles, max_splits, 128, 256]: per-split O / l
   float2* part_ml;      // [B*tiles, max_splits, 128]
   int T, H, nq, S_cap, tiles_per_req, max_splits;
+  int blocks_per_split;  // 64-key blocks per split, 1..4 (0: 4)
   int kv_row0;          // first KV row of this layer in the 2D view
   float scale_log2;     // log2(e) / sqrt(dh)
   int* err;

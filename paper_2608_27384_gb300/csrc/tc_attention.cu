@@ -8,7 +8,8 @@
 // Work decomposition.  A query tile is 128 rows = 128/nq consecutive tokens x
 // all nq heads of one request: MQA heads share the single KV head, so one K/V
 // tile in shared memory serves every head.  The key range of a tile is cut into
-// splits of 256 keys (4 blocks of 64); key blocks past the tile's largest limit
+// splits of up to 256 keys (1-4 blocks of 64: fewer when there are few query
+// tiles, so that more SMs take part); key blocks past the tile's largest limit
 // are never loaded.  One CTA handles one (tile, split):
 //   warp 0      TMA: the Q tile (64 KB) and the split's K blocks, then, once
 //               the S MMAs have read K, the V blocks into the same space;
@@ -61,14 +62,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int P = __ldg(a.prefix_len + r);
   const int limit_max = attn_key_limit(P, t_last, a.H);
   const int nkb_tile = (limit_max + kKB - 1) / kKB;
-  const int nsplit = (nkb_tile + kBlocksPerSplit - 1) / kBlocksPerSplit;
+  const int bps = a.blocks_per_split > 0 ? min(a.blocks_per_split, kBlocksPerSplit) : kBlocksPerSplit;
+  const int nsplit = (nkb_tile + bps - 1) / bps;
   if (split >= nsplit || nsplit > a.max_splits) {  // uniform over the CTA
     if (nsplit > a.max_splits && split == 0 && threadIdx.x == 0) report_error(a.err, KERR_BAD_SHAPE);
     pdl_trigger();
     return;
   }
-  const int kb0 = split * kBlocksPerSplit;
-  const int nblk = min(kBlocksPerSplit, nkb_tile - kb0);
+  const int kb0 = split * bps;
+  const int nblk = min(bps, nkb_tile - kb0);
 
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -340,7 +342,8 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
   pdl_wait();
   const int P = __ldg(a.prefix_len + r);
   const int nkb_tile = (attn_key_limit(P, t_last, a.H) + kKB - 1) / kKB;
-  const int nsplit = (nkb_tile + kBlocksPerSplit - 1) / kBlocksPerSplit;
+  const int bps = a.blocks_per_split > 0 ? min(a.blocks_per_split, kBlocksPerSplit) : kBlocksPerSplit;
+  const int nsplit = (nkb_tile + bps - 1) / bps;
   if (nsplit <= 1 || nsplit > a.max_splits) return;  // written by the attention kernel / bad size
   const size_t tbase = (size_t)(r * a.tiles_per_req + gtile) * a.max_splits;
   // the first 8 splits' partial rows are requested together with the (max, sum)
