@@ -22,21 +22,6 @@ __device__ __forceinline__ void pack_bf16x32(const float (&v)[32], uint4 (&u)[4]
   for (int i = 0; i < 4; ++i) u[i] = pack_bf16x8(&v[8 * i]);
 }
 
-// The RoPE (cos, sin) pairs the QKV epilogue of row m will read (a constant
-// table), pulled into L1 while the MMAs still run.
-template <int BN>
-__device__ __forceinline__ void gemm_epilogue_prefetch_rope(const GemmEpi& ep, int m, int M,
-                                                            int n0) {
-  if (m >= M) return;
-  const int dh = ep.dh, seg = n0 / dh, tj = (n0 % dh) / BN;
-  if (seg > ep.nq) return;  // v is not rotated
-  const int r = m / ep.T;
-  const int pos = __ldg(ep.prefix_len + r) + (m - r * ep.T);
-  const char* p = reinterpret_cast<const char*>(ep.rope + (size_t)pos * (dh / 2) + tj * (BN / 2));
-#pragma unroll
-  for (int b = 0; b < (BN / 2) * 8; b += 128) asm volatile("prefetch.global.L1 [%0];" ::"l"(p + b));
-}
-
 // This row's fp16 RoPE (cos, sin) pairs for tile column n0 (BN/2 pairs, 2*BN
 // bytes), loaded into registers while the MMAs still run; zeros where the row
 // is past M or the tile is not rotated (v).
