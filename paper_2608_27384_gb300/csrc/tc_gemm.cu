@@ -11,8 +11,11 @@
 //   warps 2..5  epilogue: tcgen05.ld of the accumulator (one TMEM lane = one
 //               output row per thread), fused post-processing, global stores.
 // Epilogues (GemmMode): bias (fp32 out), bias+SiLU (bf16 out), split-K partial
-// planes (fp32), RoPE + q / KV-workspace scatter for the packed QKV projection,
-// and tanh-GELU(gate) * up for the packed gate/up projection.
+// planes (fp32 or bf16), RoPE + q / KV-workspace scatter for the packed QKV
+// projection, and tanh-GELU(gate) * up for the packed gate/up projection.
+// Two more forms share the epilogues: a persistent weight-streaming kernel for
+// at most 16 rows (the FiLM projection) and a persistent multi-tile kernel with
+// two TMEM accumulators for shapes with many more tiles than SMs.
 // Every wait is bounded (common.cuh); on timeout the kernel records an error
 // code and finishes without touching the accumulator.
 #include "common.cuh"
