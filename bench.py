@@ -80,7 +80,7 @@ def dram_traffic(workload, kind):
 # algorithmic work per kernel launch (FLOPs, bytes)
 # ---------------------------------------------------------------------------
 
-def kernel_costs(wl, B):
+def kernel_costs(wl, B, n_sms=152):
     """Algorithmic FLOPs and DRAM bytes of one launch of each kernel kind (bf16
     weights, bf16 activations, fp32 residual stream)."""
     W, F, Dq, dh, nq, K, H, A = (wl.width, wl.mlp_dim, wl.n_q_heads * wl.head_dim,
@@ -107,8 +107,15 @@ def kernel_costs(wl, B):
     c["final_norm"] = (0.0, 4.0 * M * W * 3 + 4.0 * M * W)
     c["velocity"] = (2.0 * M * W * A, 4.0 * M * W + 4.0 * W * A + 4.0 * M * A * 3)
     tiles = -(-T * nq // 128)
-    c["attn_merge"] = (0.0, 4.0 * B * tiles * 128 * dh * max(1, -(-(max(P) + T) // 256)) +
-                       2.0 * M * Dq)
+    # the library's split of the key range: 1-4 blocks of 64 keys per split, the
+    # largest that still gives about half as many attention CTAs as SMs
+    nkb = -(-(max(P) + T) // 64)
+    bps = 4
+    while bps > 1 and B * tiles * -(-nkb // bps) < max(1, n_sms // 2):
+        bps //= 2
+    nsplit = -(-nkb // bps)
+    # bf16 partial rows (O / l) and fp32 (max, sum) read, bf16 output written
+    c["attn_merge"] = (0.0, (2.0 * dh + 8.0) * B * tiles * 128 * nsplit + 2.0 * M * Dq)
     c["timestep_embed"] = (0.0, 2.0 * BK * W)
     # fused post-attention block: O-proj, norm 2, gate/up, down, norm and (on all
     # but the last layer) the next layer's QKV; averaged over the L launches
@@ -377,7 +384,7 @@ def main():
             t, n = per_kind.get(kind, (0.0, 0))
             per_kind[kind] = (t + us, n + 1)
     prof_total = sum(t for t, _ in per_kind.values())
-    costs = kernel_costs(wl, B)
+    costs = kernel_costs(wl, B, torch.cuda.get_device_properties(dev).multi_processor_count)
     bw = peaks["hbm_gbs"] * 1e9
     tc = peaks["bf16_tflops"] * 1e12
     # The event nodes serialise the profiled graph and add a fixed cost to every
