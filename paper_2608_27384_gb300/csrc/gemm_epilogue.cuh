@@ -1,7 +1,7 @@
 // Epilogues of the tcgen05 GEMMs: one output row per thread, read from TMEM in
-// 32-column chunks and stored through a per-warp shared-memory stage with
-// coalesced 16-byte stores.  Shared by the per-op GEMM kernel and the fused
-// block kernel.
+// 32-column chunks.  bf16 rows are stored straight from registers; fp32 rows go
+// through a per-warp shared-memory stage for coalesced 16-byte stores.  Shared by
+// the per-op GEMM kernel and the fused block kernel.
 #pragma once
 
 #include <cuda_fp16.h>
@@ -9,6 +9,19 @@
 #include "kernels.h"
 
 namespace fva {
+
+// 64 bytes of one output row, straight from registers (16-byte stores): no
+// shared-memory staging, whose write and read-back would compete with the MMAs'
+// operand traffic for the SM's shared-memory bandwidth.
+__device__ __forceinline__ void store_row64(const uint4 (&u)[4], void* dst) {
+  if (dst) {
+    uint4* d = reinterpret_cast<uint4*>(dst);
+    d[0] = u[0];
+    d[1] = u[1];
+    d[2] = u[2];
+    d[3] = u[3];
+  }
+}
 
 __device__ __forceinline__ void pack_f32x32(const float (&v)[32], uint4 (&u)[8]) {
 #pragma unroll
@@ -83,15 +96,14 @@ __device__ __forceinline__ void gemm_epilogue_qkv(const GemmEpi& ep, uint32_t tr
     uint4 p1[4], p2[4];
     pack_bf16x32(x1, p1);
     pack_bf16x32(x2, p2);
-    warp_store_rows<64>(stage, p1, ok ? dst + d0 : nullptr, lane);
-    warp_store_rows<64>(stage, p2, ok ? dst + d0 + dh / 2 : nullptr, lane);
+    store_row64(p1, ok ? dst + d0 : nullptr);
+    store_row64(p2, ok ? dst + d0 + dh / 2 : nullptr);
   }
 }
 
 // Epilogue of one output row per thread; `stage` is this warp's private shared
-// memory (32 * 144 bytes): every 32-column chunk is stored through it with
-// coalesced 16-byte stores (warp_store_rows) while the next chunk is read from
-// TMEM.
+// memory (32 * 144 bytes): every 32-column fp32 chunk is stored through it with
+// coalesced 16-byte stores (warp_store_rows); bf16 chunks are stored directly.
 template <int BN, int MODE>
 __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, int m, int M,
                                               int n0, int split, uint8_t* stage, int lane) {
@@ -105,7 +117,7 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
       pack_bf16x32(v, u);
       bf16* dst = ok ? (bf16*)ep.out + split * ep.split_stride + (size_t)m * ep.ldo + n0 + c
                      : nullptr;
-      warp_store_rows<64>(stage, u, dst, lane);
+      store_row64(u, dst);
     }
   } else if constexpr (MODE == GEMM_BIAS_F32 || MODE == GEMM_BIAS_SILU_BF16 ||
                        MODE == GEMM_PARTIAL_F32) {
@@ -133,8 +145,7 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
         } else {
           uint4 u[4];
           pack_bf16x32(v, u);
-          warp_store_rows<64>(stage, u, ok ? (bf16*)ep.out + (size_t)m * ep.ldo + n0 + c : nullptr,
-                              lane);
+          store_row64(u, ok ? (bf16*)ep.out + (size_t)m * ep.ldo + n0 + c : nullptr);
         }
       }
     }
@@ -150,8 +161,7 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
       for (int i = 0; i < 32; ++i) g[i] = gelu_tanh_f(g[i]) * u[i];
       uint4 pk[4];
       pack_bf16x32(g, pk);
-      warp_store_rows<64>(stage, pk, ok ? (bf16*)ep.out + (size_t)m * ep.ldo + n0 / 2 + c : nullptr,
-                          lane);
+      store_row64(pk, ok ? (bf16*)ep.out + (size_t)m * ep.ldo + n0 / 2 + c : nullptr);
     }
   } else if constexpr (MODE == GEMM_QKV_ROPE) {
     // Weight rows are permuted so that tile column c < BN/2 holds head dim
@@ -197,8 +207,8 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
       uint4 p1[4], p2[4];
       pack_bf16x32(x1, p1);
       pack_bf16x32(x2, p2);
-      warp_store_rows<64>(stage, p1, ok ? dst + d0 : nullptr, lane);
-      warp_store_rows<64>(stage, p2, ok ? dst + d0 + dh / 2 : nullptr, lane);
+      store_row64(p1, ok ? dst + d0 : nullptr);
+      store_row64(p2, ok ? dst + d0 + dh / 2 : nullptr);
     }
   }
 }
