@@ -56,7 +56,7 @@ def load_peaks():
 
 def dram_traffic(workload, kind):
     """DRAM bytes (read + write) per launch of `kind` from the committed ncu
-    summary, if it was taken on this workload with the kernel source unchanged
+    summary, if it was taken on this workload with the kernel's sources unchanged
     since (else None)."""
     path = os.path.join(ROOT, "profiles", "dram_traffic.json")
     try:
@@ -67,13 +67,15 @@ def dram_traffic(workload, kind):
     e = tab.get(workload, {}).get(kind)
     if not e:
         return None
-    src = os.path.join(ROOT, e["source"])
-    try:
-        with open(src, "rb") as f:
-            digest = hashlib.sha256(f.read()).hexdigest()
-    except OSError:
-        return None
-    return e["dram_bytes_per_launch"] if digest == e["source_sha256"] else None
+    sources = e.get("sources") or {e["source"]: e["source_sha256"]}
+    for rel, want in sources.items():
+        try:
+            with open(os.path.join(ROOT, rel), "rb") as f:
+                if hashlib.sha256(f.read()).hexdigest() != want:
+                    return None
+        except OSError:
+            return None
+    return e["dram_bytes_per_launch"]
 
 
 # ---------------------------------------------------------------------------
