@@ -866,6 +866,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   d.S_cap = h->S_cap;
   d.N_mod = h->N_mod;
   d.eps = h->cfg.rms_eps;
+  d.n_sms = h->n_sms;
   const int M = B * h->T, BK = B * h->K, W = h->W, F = h->F, Dq = h->Dq, L = h->L;
   const bool bf = h->bf16;
   const size_t a = h->act;

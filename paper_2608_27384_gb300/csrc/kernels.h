@@ -23,6 +23,7 @@ struct StepDims {
   int S_cap;   // KV rows per request and layer: max_prefix + T
   int N_mod;   // FiLM outputs per chunk: L*6W + 2W
   float eps;
+  int n_sms;   // SMs of the device (launch-shape choices; 0: unknown)
 };
 
 // FiLM slice offsets inside one row of `mod` [B*K, N_mod].

@@ -354,23 +354,13 @@ __global__ void __launch_bounds__(256)
   }
 }
 
-static int device_sms() {
-  static int n = [] {
-    int dev = 0, v = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
-    return v > 0 ? v : 1;
-  }();
-  return n;
-}
-
 template <typename Part>
 static void launch_resid_norm_t(const StepDims& d, int rows, float* h, const Part* part,
                                 int n_parts, long long part_stride, const float* mod,
                                 int gate_off, int scale_off, int shift_off, void* y,
                                 bool act_bf16, cudaStream_t s) {
   constexpr int R = 4;
-  if (d.W == 1024 && n_parts <= 2 && rows >= R * 4 * device_sms()) {
+  if (d.W == 1024 && n_parts <= 2 && d.n_sms > 0 && rows >= R * 4 * d.n_sms) {
     const dim3 grid((rows + R - 1) / R);
     if (act_bf16)
       launch_pdl(resid_norm_rows_kernel<bf16, Part, R>, grid, dim3(256), 0, s, d, rows, h, part,
