@@ -286,7 +286,7 @@ __device__ __forceinline__ void epi_geglu(const GemmEpi& ep, uint32_t trow, int 
     tmem_ld_wait();
     float o[32];
 #pragma unroll
-    for (int i = 0; i < 32; ++i) o[i] = gelu_tanh_f(__uint_as_float(g[i])) * __uint_as_float(u[i]);
+    for (int i = 0; i < 32; ++i) o[i] = gelu_tanh_bf16out(__uint_as_float(g[i])) * __uint_as_float(u[i]);
     uint4 pk[4];
     pack_bf16x32(o, pk);
     warp_store_rows<64>(stage, pk, ok ? (bf16*)ep.out + (size_t)m * ep.ldo + n0 / 2 + c : nullptr,

@@ -158,7 +158,7 @@ __device__ __forceinline__ void gemm_epilogue(const GemmEpi& ep, uint32_t trow, 
       tmem_ld32(trow + c, g);
       tmem_ld32(trow + half + c, u);
 #pragma unroll
-      for (int i = 0; i < 32; ++i) g[i] = gelu_tanh_f(g[i]) * u[i];
+      for (int i = 0; i < 32; ++i) g[i] = gelu_tanh_bf16out(g[i]) * u[i];
       uint4 pk[4];
       pack_bf16x32(g, pk);
       store_row64(pk, ok ? (bf16*)ep.out + (size_t)m * ep.ldo + n0 / 2 + c : nullptr);
