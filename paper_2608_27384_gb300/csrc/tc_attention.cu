@@ -1,4 +1,7 @@
-// Chunk-wise causal multi-query attention on tcgen05 (head_dim 256, bf16).
+// Chunk-wise causal multi-query attention on tcgen05 (head_dim 256, bf16), split-KV
+// form with global scratch.  The step uses attn_cluster_kernel (attention_cluster.cu),
+// which combines its key splits inside a thread-block cluster; this form serves
+// fva_chunk_attention_noalloc, whose scratch is a fixed device array.
 //
 // The paper's mask (§3.1): action token t of chunk c(t) = floor(t / H) attends to
 // every prefix key of its request and to the action keys of chunks <= c(t)
@@ -64,8 +67,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int nkb_tile = (limit_max + kKB - 1) / kKB;
   const int bps = a.blocks_per_split > 0 ? min(a.blocks_per_split, kBlocksPerSplit) : kBlocksPerSplit;
   const int nsplit = (nkb_tile + bps - 1) / bps;
-  if (split >= nsplit || nsplit > a.max_splits) {  // uniform over the CTA
-    if (nsplit > a.max_splits && split == 0 && threadIdx.x == 0) report_error(a.err, KERR_BAD_SHAPE);
+  // a prefix length the KV rows cannot hold (its keys would run into the next
+  // request's rows) or more splits than the scratch holds: the tile is left
+  // unwritten and the error word records it
+  const bool bad = P < 0 || P + a.T > a.S_cap || nsplit > a.max_splits;
+  if (split >= nsplit || bad) {  // uniform over the CTA
+    if (bad && split == 0 && threadIdx.x == 0) report_error(a.err, KERR_BAD_SHAPE);
     pdl_trigger();
     return;
   }
@@ -148,7 +155,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t idesc_s = umma_idesc_bf16(kRows, nblk * kKB, false);
     constexpr uint32_t idesc_o = umma_idesc_bf16(kRows, kDH, true);
     constexpr uint32_t kSlabK = kBlocksPerSplit * kKB * 128;  // 32 KB between head-dim slabs
-    const uint32_t qp_base = smem_u32(sQP), kv_base = smem_u32(sKV);
+    const uint64_t qd0 = umma_desc_sw128(smem_u32(sQP), 16, 1024);
+    const uint64_t kd0 = umma_desc_sw128(smem_u32(sKV), 16, 1024);
     bool good = true;
     for (int j = 0; good && j < 4; ++j) {  // head-dim slab j: 4 steps of 16
       if (!mbar_wait(&qk_full[j], 0, a.err, KERR_WAIT_TMA)) {
@@ -156,18 +164,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       tc_fence_after();
+      const uint64_t ad = desc_advance(qd0, j * (kRows * 128));
+      const uint64_t bd = desc_advance(kd0, j * kSlabK);
 #pragma unroll
-      for (int kk = 0; kk < 4; ++kk) {
-        const uint32_t off = kk * 32;  // 16 bf16 along K inside the 128-byte row
-        const uint64_t ad = umma_desc_sw128(qp_base + j * (kRows * 128) + off, 16, 1024);
-        const uint64_t bd = umma_desc_sw128(kv_base + j * kSlabK + off, 16, 1024);
-        umma_bf16(tS, ad, bd, idesc_s, (j > 0 || kk > 0) ? 1u : 0u);
-      }
+      for (int kk = 0; kk < 4; ++kk)  // 16 bf16 = 32 bytes along K inside the 128-byte row
+        umma_bf16(tS, ad + 2 * kk, bd + 2 * kk, idesc_s, (j > 0 || kk > 0) ? 1u : 0u);
     }
     if (good) {
       umma_commit(k_free);
       umma_commit(s_full);
     }
+    const uint64_t vd0 = umma_desc_sw128(smem_u32(sKV), kSlabK, 1024);
     for (int j = 0; good && j < nblk; ++j) {
       // block j's P (written while the softmax threads still work on later
       // blocks) and V
@@ -177,14 +184,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       tc_fence_after();
+      // P keys j*64 + 16 ks .. +15 from TMEM (bf16 pairs, 8 columns); V the same
+      // keys, all 256 head dims: MN-major B operand whose 64-wide head-dim slabs
+      // are kSlabK apart (16 keys = 2 KB further on per step).
+      const uint64_t bv = desc_advance(vd0, j * kKB * 128);
 #pragma unroll
-      for (int ks = 0; ks < kKB / 16; ++ks) {
-        // P keys j*64 + 16 ks .. +15 from TMEM (bf16 pairs, 8 columns); V the same
-        // keys, all 256 head dims: MN-major B operand whose 64-wide head-dim slabs
-        // are kSlabK apart.
-        const uint64_t bd = umma_desc_sw128(kv_base + (j * kKB + ks * 16) * 128, kSlabK, 1024);
-        umma_bf16_ts(tO, tS + j * (kKB / 2) + ks * 8, bd, idesc_o, (j > 0 || ks > 0) ? 1u : 0u);
-      }
+      for (int ks = 0; ks < kKB / 16; ++ks)
+        umma_bf16_ts(tO, tS + j * (kKB / 2) + ks * 8, bv + 128 * ks, idesc_o,
+                     (j > 0 || ks > 0) ? 1u : 0u);
     }
     if (good) umma_commit(o_full);
   } else if (warp >= 2) {
@@ -344,7 +351,8 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
   const int nkb_tile = (attn_key_limit(P, t_last, a.H) + kKB - 1) / kKB;
   const int bps = a.blocks_per_split > 0 ? min(a.blocks_per_split, kBlocksPerSplit) : kBlocksPerSplit;
   const int nsplit = (nkb_tile + bps - 1) / bps;
-  if (nsplit <= 1 || nsplit > a.max_splits) return;  // written by the attention kernel / bad size
+  // written by the attention kernel, or a bad size it left unwritten
+  if (nsplit <= 1 || nsplit > a.max_splits || P < 0 || P + a.T > a.S_cap) return;
   const size_t tbase = (size_t)(r * a.tiles_per_req + gtile) * a.max_splits;
   // the first 8 splits' partial rows are requested together with the (max, sum)
   // pairs, so both round trips overlap

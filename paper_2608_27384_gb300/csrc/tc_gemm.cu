@@ -105,24 +105,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer
     constexpr uint32_t idesc = umma_idesc_bf16(kBM, BN, false);
+    const uint64_t d0 = umma_desc_sw128(smem_u32(smem), 16, 1024);  // A of stage 0
     bool good = true;
+    int s = 0;
+    uint32_t ph = 0;
     for (int i = 0; i < nkb; ++i) {
-      const int s = i % C::kStages;
-      const uint32_t ph = (uint32_t)(i / C::kStages) & 1u;
       if (!mbar_wait(&full[s], ph, ep.err, KERR_WAIT_TMA)) {
         good = false;
         break;
       }
       tc_fence_after();
-      const uint32_t sa = smem_u32(smem + s * C::kStageBytes);
-      const uint32_t sb = sa + C::kABytes;
+      const uint64_t ad = desc_advance(d0, s * C::kStageBytes);
+      const uint64_t bd = desc_advance(ad, C::kABytes);
 #pragma unroll
-      for (int kk = 0; kk < kBK / 16; ++kk) {
-        const uint64_t ad = umma_desc_sw128(sa + kk * 32, 16, 1024);
-        const uint64_t bd = umma_desc_sw128(sb + kk * 32, 16, 1024);
-        umma_bf16(tmem, ad, bd, idesc, (i > 0 || kk > 0) ? 1u : 0u);
-      }
+      for (int kk = 0; kk < kBK / 16; ++kk)  // 16 bf16 = 32 bytes along K per step
+        umma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (i > 0 || kk > 0) ? 1u : 0u);
       umma_commit(&empty[s]);
+      if (++s == C::kStages) {
+        s = 0;
+        ph ^= 1u;
+      }
     }
     if (good) umma_commit(acc_full);
   } else if (warp >= 2) {
@@ -253,7 +255,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer
     constexpr uint32_t idesc = umma_idesc_bf16(kBM, BN, false);
-    uint32_t it = 0, acc = 0;
+    const uint64_t d0 = umma_desc_sw128(smem_u32(smem), 16, 1024);  // A of stage 0
+    uint32_t it = 0, acc = 0, rph = 0;
+    int rs = 0;
     bool ok = true;
     for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x, ++acc) {
       const uint32_t buf = acc & 1u;
@@ -261,21 +265,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const uint32_t d = tmem + buf * BN;
       for (int i = 0; i < nkb; ++i, ++it) {
-        const int s = it % C::kStages;
-        if (!mbar_wait(&full[s], (it / C::kStages) & 1u, ep.err, KERR_WAIT_TMA)) {
+        if (!mbar_wait(&full[rs], rph, ep.err, KERR_WAIT_TMA)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t sa = smem_u32(smem + s * C::kStageBytes);
-        const uint32_t sb = sa + C::kABytes;
+        const uint64_t ad = desc_advance(d0, rs * C::kStageBytes);
+        const uint64_t bd = desc_advance(ad, C::kABytes);
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk) {
-          const uint64_t ad = umma_desc_sw128(sa + kk * 32, 16, 1024);
-          const uint64_t bd = umma_desc_sw128(sb + kk * 32, 16, 1024);
-          umma_bf16(d, ad, bd, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+        for (int kk = 0; kk < kBK / 16; ++kk)  // 16 bf16 = 32 bytes along K per step
+          umma_bf16(d, ad + 2 * kk, bd + 2 * kk, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+        umma_commit(&empty[rs]);
+        if (++rs == C::kStages) {
+          rs = 0;
+          rph ^= 1u;
         }
-        umma_commit(&empty[s]);
       }
       if (ok) umma_commit(&acc_full[buf]);
     }
@@ -405,7 +409,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer
     constexpr uint32_t idesc = umma_idesc_bf16(kBM, BN, false);
-    uint32_t it = 0, acc = 0;
+    const uint64_t d0 = umma_desc_sw128(smem_u32(smem), 16, 1024);  // A of stage 0
+    uint32_t it = 0, acc = 0, rph = 0;
+    int rs = 0;
     bool ok = true;
     for (int t = blockIdx.x; ok && t < tiles; t += gridDim.x, ++acc) {
       const uint32_t buf = acc & 1u;
@@ -413,21 +419,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const uint32_t d = tmem + buf * BN;
       for (int i = 0; i < nkb; ++i, ++it) {
-        const int s = it % C::kStages;
-        if (!mbar_wait(&full[s], (it / C::kStages) & 1u, ep.err, KERR_WAIT_TMA)) {
+        if (!mbar_wait(&full[rs], rph, ep.err, KERR_WAIT_TMA)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t sa = smem_u32(smem + s * C::kStageBytes);
-        const uint32_t sb = sa + C::kABytes;
+        const uint64_t ad = desc_advance(d0, rs * C::kStageBytes);
+        const uint64_t bd = desc_advance(ad, C::kABytes);
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk) {
-          const uint64_t ad = umma_desc_sw128(sa + kk * 32, 16, 1024);
-          const uint64_t bd = umma_desc_sw128(sb + kk * 32, 16, 1024);
-          umma_bf16(d, ad, bd, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+        for (int kk = 0; kk < kBK / 16; ++kk)  // 16 bf16 = 32 bytes along K per step
+          umma_bf16(d, ad + 2 * kk, bd + 2 * kk, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+        umma_commit(&empty[rs]);
+        if (++rs == C::kStages) {
+          rs = 0;
+          rph ^= 1u;
         }
-        umma_commit(&empty[s]);
       }
       if (ok) umma_commit(&acc_full[buf]);
     }
