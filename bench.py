@@ -119,11 +119,6 @@ def kernel_costs(wl, B, n_sms=152):
     # bf16 partial rows (O / l) and fp32 (max, sum) read, bf16 output written
     c["attn_merge"] = (0.0, (2.0 * dh + 8.0) * B * tiles * 128 * nsplit + 2.0 * M * Dq)
     c["timestep_embed"] = (0.0, 2.0 * BK * W)
-    # fused post-attention block: O-proj, norm 2, gate/up, down, norm and (on all
-    # but the last layer) the next layer's QKV; averaged over the L launches
-    nxt = (L - 1) / L
-    c["block"] = tuple(c["out_proj"][i] + c["gate_up"][i] + c["down"][i] +
-                       2 * c["resid_norm"][i] + nxt * c["qkv"][i] for i in range(2))
     return c
 
 

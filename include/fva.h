@@ -60,6 +60,11 @@ typedef enum fva_dtype {
  * no-causal ablation of the paper's App. A.3) instead of the chunk-causal mask of
  * Sec. 3.1. */
 #define FVA_FLAG_BLOCK_DIAGONAL 2u
+/* bf16: run every projection as one launch of per-tile CTAs, never in the persistent
+ * form (one CTA per SM walking several output tiles with two TMEM accumulators) that
+ * is otherwise used where a projection has at least two output tiles per SM (large
+ * batches).  Both forms give bit-identical results. */
+#define FVA_FLAG_NO_PERSISTENT_GEMM 4u
 
 /*
  * Shape and numerics of the action expert and of the streaming buffer.
@@ -104,14 +109,8 @@ typedef struct fva_handle fva_handle;
  * device buffer for max_batch requests (weights, prefix/action K/V workspace,
  * activations, scratch) and zero-fills them.  *out receives the handle.
  * Errors: INVALID_ARG (bad field), UNSUPPORTED (shape outside the dtype's
- * kernels), OOM, CUDA.  Nothing is allocated when an error is returned.
- * Environment: FVA_BLOCK_KERNEL=1 (read here) makes bf16 steps run each layer's
- * post-attention part as one persistent kernel (FVA_K_BLOCK) instead of one
- * launch per operation, where the sizes allow it (width a multiple of 256 up to
- * 1024); results agree within the bf16 tolerances, not bit for bit.
- * FVA_GEMM_PERSIST=0 (read here) turns off the persistent form of the bf16
- * projections, which is otherwise used when a projection has at least two output
- * tiles per SM and no K-split (large batches); both forms give identical results.
+ * kernels), OOM, CUDA.  Nothing is allocated when an error is returned.  No
+ * environment variable is read.
  */
 fva_status fva_create(const fva_config* cfg, fva_handle** out);
 
@@ -298,9 +297,7 @@ typedef enum fva_kernel_kind {
   FVA_K_FINAL = 10,          /* last gated residual + final FiLM RMSNorm (fp32 out)  */
   FVA_K_ATTN_MERGE = 11,     /* combination of the attention's key splits            */
   FVA_K_VELOCITY = 12,       /* out-projection + Euler + emit + roll + tail          */
-  FVA_K_BLOCK = 13,          /* fused post-attention part of a layer: O-projection,
-                                norm 2, gate/up, down, then the next layer's norm 1
-                                and QKV projection (or the final norm)               */
+  FVA_K_BLOCK = 13,          /* reserved (no longer launched)                        */
   FVA_K_COUNT = 14
 } fva_kernel_kind;
 

@@ -22,6 +22,7 @@ FVA_ABI_VERSION = 1
 FVA_FP32, FVA_BF16 = 0, 1
 FVA_FLAG_NO_GRAPH = 1
 FVA_FLAG_BLOCK_DIAGONAL = 2
+FVA_FLAG_NO_PERSISTENT_GEMM = 4
 FVA_PARAM_RING = 8
 
 STATUS = {0: "FVA_OK", 1: "FVA_ERR_INVALID_ARG", 2: "FVA_ERR_STATE", 3: "FVA_ERR_OOM",
@@ -61,7 +62,7 @@ class fva_kernel_time(ctypes.Structure):
 
 KERNEL_KINDS = ["timestep_embed", "time_mlp", "film", "embed_norm", "qkv", "attention",
                 "out_proj", "resid_norm", "gate_up", "down", "final_norm", "attn_merge",
-                "velocity", "block"]
+                "velocity", "reserved_13"]
 
 EXPORTS = ["fva_create", "fva_destroy", "fva_num_weights", "fva_weight_shape",
            "fva_load_weights", "fva_set_prefix_kv", "fva_step", "fva_step_ex",

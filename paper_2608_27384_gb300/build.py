@@ -19,7 +19,7 @@ BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libfva.so")
 
 SOURCES = ["fva_api.cu", "rowwise.cu", "tc_gemm.cu", "tc_attention.cu", "simt_f32.cu",
-           "attention_noalloc.cu", "block_kernel.cu"]
+           "attention_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

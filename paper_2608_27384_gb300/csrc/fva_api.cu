@@ -128,15 +128,10 @@ struct fva_handle {
   int W, nq, dh, Dq, F, A, K, H, T, L, Bmax, Pmax, S_cap, N_qkv, N_mod, BKmax, Mmax;
   int tiles_per_req = 0, attn_max_splits = 0, attn_bps = 4;
   int n_sms = 0;
-  // fused post-attention block kernel (bf16): task lists per batch size
-  bool block_on = false;
   int bn_qkv = kBnQKV, bn_gu = kBnGU;  // tile widths of the QKV and gate/up weight layouts
-  bool persist_on = true;  // persistent GEMMs where tiles >= 2 x SMs (FVA_GEMM_PERSIST=0: off)
-  int blk_split_o = 1, blk_split_d = 1;
-  BlockTask* blk_tasks = nullptr;
-  std::vector<int> blk_off, blk_n;  // [2 * (B - 1) + last]
-  unsigned* blk_ctr = nullptr;      // [L][m_tiles_max * kBlockCtrPerTile]
-  size_t blk_ctr_layer = 0;
+  // persistent GEMMs where a projection has at least two tiles per SM
+  // (FVA_FLAG_NO_PERSISTENT_GEMM: off)
+  bool persist_on = true;
 
   std::vector<void*> allocs;
   // weights
@@ -263,7 +258,7 @@ fva_status validate_config(const fva_config* c) {
       !std::isfinite(c->rope_theta))
     return fail(FVA_ERR_INVALID_ARG, "bad rms_eps / rope_theta / timestep periods");
   if (c->action_dim > 128) return fail(FVA_ERR_UNSUPPORTED, "action_dim > 128");
-  if (c->flags & ~(FVA_FLAG_NO_GRAPH | FVA_FLAG_BLOCK_DIAGONAL))
+  if (c->flags & ~(FVA_FLAG_NO_GRAPH | FVA_FLAG_BLOCK_DIAGONAL | FVA_FLAG_NO_PERSISTENT_GEMM))
     return fail(FVA_ERR_INVALID_ARG, "unknown flags 0x%x", c->flags);
   const long long T = (long long)c->n_chunks * c->chunk_tokens;
   if (T * c->max_batch > (1LL << 24) || c->max_prefix > (1 << 20) || c->n_layers > 1024)
@@ -360,7 +355,6 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
     CUDA_TRY(tc_attention_init());
     if (h->W > 4096) return fail(FVA_ERR_UNSUPPORTED, "bf16 kernels need width <= 4096");
     CUDA_TRY(gemv_init(h->W));
-    CUDA_TRY(block_kernel_init());
     CUDA_TRY(cudaDeviceGetAttribute(&h->n_sms, cudaDevAttrMultiProcessorCount, h->device));
   }
   const size_t a = h->act;
@@ -393,55 +387,11 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
     }
   }
   if (h->bf16) {
-    // K-splits of the block kernel's output and down projections: 4 where the
-    // sizes allow it (tasks of 8-16 k-blocks of 64)
-    auto pick = [](int kblocks, int F) {
-      for (int s : {4, 2, 1})
-        if (kblocks % s == 0 && (F == 0 || F % (s * 128) == 0)) return s;
-      return 1;
-    };
-    h->blk_split_o = pick(h->Dq / 64, 0);
-    h->blk_split_d = pick(h->F / 64, h->F);
     if (h->Mmax <= 128) {  // one row tile: narrower QKV and gate/up tiles
       h->bn_qkv = kBnSmall;
       h->bn_gu = kBnSmall;
     }
-    const char* penv = std::getenv("FVA_GEMM_PERSIST");
-    h->persist_on = !(penv && penv[0] == '0');
-    // opt-in (FVA_BLOCK_KERNEL=1): on the 500-token workloads the per-operation
-    // kernels are faster (every stage of the block kernel still waits for the
-    // previous one, and its early weight prefetch competes with epilogue stores
-    // for the SM's memory port)
-    const char* env = std::getenv("FVA_BLOCK_KERNEL");
-    const bool wanted = env && env[0] == '1';
-    BlockShape bs{h->Mmax, h->W, h->F, h->Dq, h->N_qkv, h->blk_split_o, h->blk_split_d, true};
-    h->block_on = wanted && h->n_sms > 0 && h->bn_gu == kBnGU && h->bn_qkv == kBnQKV &&
-                  block_supported(bs);
-    if (h->block_on) {
-      std::vector<BlockTask> all;
-      h->blk_off.assign(2 * h->Bmax, 0);
-      h->blk_n.assign(2 * h->Bmax, 0);
-      for (int B = 1; B <= h->Bmax; ++B)
-        for (int last = 0; last < 2; ++last) {
-          bs.M = B * h->T;
-          bs.next_qkv = last == 0;
-          const int mx = block_max_tasks(bs);
-          const size_t off = all.size();
-          all.resize(off + mx);
-          int n = 0;
-          build_block_tasks(bs, all.data() + off, &n, mx);
-          all.resize(off + n);
-          h->blk_off[2 * (B - 1) + last] = (int)off;
-          h->blk_n[2 * (B - 1) + last] = n;
-        }
-      if ((st = dalloc(h, &h->blk_tasks, all.size()))) return st;
-      CUDA_TRY(cudaMemcpy(h->blk_tasks, all.data(), all.size() * sizeof(BlockTask),
-                          cudaMemcpyHostToDevice));
-      h->blk_ctr_layer = (size_t)((h->Mmax + 127) / 128) * kBlockCtrPerTile;
-      if ((st = dalloc(h, &h->blk_ctr, h->blk_ctr_layer * h->L))) return st;
-      part_elems = std::max(part_elems, (size_t)std::max(h->blk_split_o, h->blk_split_d) *
-                                            h->Mmax * h->W);
-    }
+    h->persist_on = !(c.flags & FVA_FLAG_NO_PERSISTENT_GEMM);
   }
   if ((st = dalloc(h, &h->part, part_elems))) return st;
   if (!h->bf16) {
@@ -884,11 +834,6 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     return cudaMemcpyAsync(tr_at(off), h->h, MW * 4, cudaMemcpyDeviceToDevice, s);
   };
 
-  // the fused block kernel covers each layer's post-attention part (not when a
-  // layer's intermediate tensors are traced: they stay inside that kernel)
-  const bool blk = bf && h->block_on && tr.layer < 0;
-  if (blk)
-    CUDA_TRY(cudaMemsetAsync(h->blk_ctr, 0, h->blk_ctr_layer * L * sizeof(unsigned), s));
 
   // ---- per-chunk FiLM condition and modulation (App. A.4)
   mark(FVA_K_TIMESTEP_EMBED, -1);
@@ -960,10 +905,8 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       CUDA_TRY(copy_h(o_hin));
       launch_to_f32(h->y, bf, tr_at(o_y1), (long long)MW, s);
     }
-    // QKV projection + RoPE + KV append (from layer 1 on, the block kernel of the
-    // previous layer computes it)
-    if (blk && l > 0) {
-    } else if (bf) {
+    // QKV projection + RoPE + KV append
+    if (bf) {
       ep = GemmEpi{};
       ep.err = h->err_dev;
       ep.q = h->q;
@@ -1019,59 +962,6 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
                            (float*)h->attn, B, h->T, h->H, h->nq, h->dh, h->S_cap, h->S_cap, s);
     }
     if (trace) launch_to_f32(h->attn, bf, tr_at(o_att), (long long)M * Dq, s);
-    if (blk) {
-      const bool last = l + 1 == L;
-      const LayerW& nx = h->layers[last ? l : l + 1];
-      BlockShape bs{M, W, F, Dq, h->N_qkv, h->blk_split_o, h->blk_split_d, !last};
-      BlockLaunch bl{};
-      bl.a[0] = &h->m_attn;
-      bl.a[1] = &h->m_y;
-      bl.a[2] = &h->m_mlp;
-      bl.a[3] = &h->m_y;
-      bl.b[0] = &lw.m_o;
-      bl.b[1] = &lw.m_gu;
-      bl.b[2] = &lw.m_d;
-      bl.b[3] = &nx.m_qkv;
-      bl.b_box[0] = kBnResid;
-      bl.b_box[1] = kBnGU;
-      bl.b_box[2] = kBnResid;
-      bl.b_box[3] = kBnQKV;
-      for (int i = 0; i < 4; ++i) bl.epi[i].err = h->err_dev;
-      bl.epi[0].out = h->part;
-      bl.epi[0].ldo = W;
-      bl.epi[0].split_stride = pstride;
-      bl.epi[1].out = h->mlp;
-      bl.epi[1].ldo = F;
-      bl.epi[2] = bl.epi[0];
-      GemmEpi& eq = bl.epi[3];
-      eq.q = h->q;
-      eq.kc = (uint8_t*)h->kc + (size_t)(last ? l : l + 1) * kv_layer * a;
-      eq.vc = (uint8_t*)h->vc + (size_t)(last ? l : l + 1) * kv_layer * a;
-      eq.prefix_len = h->prefix_len_dev;
-      eq.rope = h->rope;
-      eq.rope_h = h->rope_h;
-      eq.T = h->T;
-      eq.S_cap = h->S_cap;
-      eq.nq = h->nq;
-      eq.dh = h->dh;
-      bl.norm[0] = BlockNorm{h->h, h->part, h->blk_split_o, pstride, h->mod, mod_off(l, 2, W),
-                             mod_off(l, 3, W), mod_off(l, 4, W), h->y, 0};
-      if (!last)
-        bl.norm[1] = BlockNorm{h->h, h->part, h->blk_split_d, pstride, h->mod, mod_off(l, 5, W),
-                               mod_off(l + 1, 0, W), mod_off(l + 1, 1, W), h->y, 0};
-      else
-        bl.norm[1] = BlockNorm{h->h, h->part, h->blk_split_d, pstride, h->mod, mod_off(l, 5, W),
-                               modf_off(L, 0, W), modf_off(L, 1, W), h->yF, 1};
-      bl.d = d;
-      const int li = 2 * (B - 1) + (last ? 1 : 0);
-      bl.tasks = h->blk_tasks + h->blk_off[li];
-      bl.n_tasks = h->blk_n[li];
-      bl.ctr = h->blk_ctr + (size_t)l * h->blk_ctr_layer;
-      bl.err = h->err_dev;
-      mark(FVA_K_BLOCK, l);
-      CUDA_TRY(launch_block_kernel(bs, bl, h->n_sms, s));
-      continue;
-    }
     // output projection (split-K partials) -> gated residual + norm 2
     if (bf) {
       ep = GemmEpi{};
@@ -1118,7 +1008,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     }
   }
   // ---- final norm, out-projection, Euler update, emit, roll, tail
-  if (!blk) {
+  {
     mark(FVA_K_FINAL, -1);
     launch_final_norm(d, h->h, h->part, bf, sp_d, pstride, h->mod, h->yF, s);
   }

@@ -173,70 +173,6 @@ cudaError_t launch_tc_attention(const CUtensorMap* q, const CUtensorMap* k,
                                 const CUtensorMap* v, const AttnArgs& a, int B,
                                 cudaStream_t s);
 
-// ---------------------------------------------------------------- block_kernel.cu
-// The part of a layer after attention (output projection, gated residual,
-// norm 2, gate/up, down, gated residual, and then either the next layer's
-// norm 1 + QKV projection or the final norm) as one persistent kernel that
-// walks a task list.  Tasks wait on per-row-tile counters that earlier tasks
-// raise, so a row tile moves to its next stage as soon as its inputs exist.
-enum BlockTaskKind : uint16_t {
-  BK_OUT_PROJ = 0,   // m, n, split: attn x W_o^T (K-slice) -> part[split]
-  BK_NORM_MID = 1,   // rows [m, m + n): h += g1 * sum part; y = norm2(h)
-  BK_GATE_UP = 2,    // m, n: y x W_gu^T -> gelu(gate) * up -> mlp
-  BK_DOWN = 3,       // m, n, split: mlp x W_d^T (K-slice) -> part[split]
-  BK_NORM_NEXT = 4,  // rows [m, m + n): h += g2 * sum part; y = next norm (or final norm)
-  BK_QKV = 5,        // m, n: y x W_qkv^T -> RoPE -> q, KV workspace (next layer)
-};
-
-struct BlockTask {
-  uint16_t kind, m, n, split;
-  uint16_t wait_ctr, wait_target;  // counter index / value to wait for (0xffff: none)
-  uint16_t done_ctr, pad;          // counter raised when done (0xffff: none)
-};
-constexpr uint16_t kNoCounter = 0xffff;
-
-// Counters of one launch: kBlockCtrPerTile per 128-row tile.
-constexpr int kBlockCtrPerTile = 16;
-constexpr int kBlockMaxSplits = 8;
-
-struct BlockShape {
-  int M, W, F, Dq, N_qkv;
-  int split_o, split_d;  // K-splits of the output and down projections
-  bool next_qkv;         // false on the last layer (final norm instead of norm 1 + QKV)
-};
-// Whether the block kernel supports these sizes (else the per-op kernels run).
-bool block_supported(const BlockShape& s);
-// Task list of one launch (same for every layer of a step with this shape).
-void build_block_tasks(const BlockShape& s, BlockTask* out, int* n_tasks, int max_tasks);
-int block_max_tasks(const BlockShape& s);
-
-struct BlockNorm {
-  float* h;
-  const float* part;
-  int n_parts;
-  long long part_stride;
-  const float* mod;
-  int gate_off, scale_off, shift_off;
-  void* y;
-  int y_f32;
-};
-
-struct BlockLaunch {
-  const CUtensorMap* a[4];  // activations: attn, y, mlp, y
-  const CUtensorMap* b[4];  // weights: W_o, W_gu, W_d, next layer's W_qkv
-  int b_box[4];             // rows of one TMA box of each weight map
-  GemmEpi epi[4];
-  BlockNorm norm[2];        // BK_NORM_MID, BK_NORM_NEXT
-  StepDims d;
-  const BlockTask* tasks;
-  int n_tasks;
-  unsigned* ctr;            // this launch's counters, zero on entry
-  int* err;
-};
-cudaError_t block_kernel_init();
-cudaError_t launch_block_kernel(const BlockShape& s, const BlockLaunch& l, int grid,
-                                cudaStream_t st);
-
 // ---------------------------------------------------------------- simt_f32.cu
 // C[M, N] = A[M, K] (lda) * B[N, K]^T, fp32 on CUDA cores.
 void launch_f32_gemm(const float* A, int lda, const float* B, float* C, int ldc, int M, int N,

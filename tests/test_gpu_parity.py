@@ -59,31 +59,6 @@ def test_small_bf16_step(name):
         case.close()
 
 
-@pytest.mark.parametrize("name", ["base", "multi_split", "batch3_ragged"])
-def test_small_bf16_step_block_kernel(name, monkeypatch):
-    """The same steps with the fused post-attention block kernel switched on, and
-    the two schedules against each other."""
-    import paper_2608_27384_gb300 as fva
-    wl = WL.small_bf16_workload(**SMALL_BF16[name])
-    fresh = WL.make_fresh_noise(wl, 1)[0]
-    results = {}
-    for mode in ("1", "0"):
-        monkeypatch.setenv("FVA_BLOCK_KERNEL", mode)
-        case = Case(wl)
-        try:
-            results[mode] = case.run(fresh=fresh)
-            if mode == "1":
-                check_step(case, results[mode], case.oracle_step(fresh=fresh), "bf16")
-            kinds = [k for k, _, _ in fva.fva_step_profile(
-                case.handle, case.dev(case.buf), case.tau,
-                case.torch.empty((wl.batch, wl.chunk_tokens, wl.action_dim), device="cuda"),
-                wl.batch)]
-            assert ("block" in kinds) == (mode == "1"), kinds
-        finally:
-            case.close()
-    assert_close(results["1"]["vel"], results["0"]["vel"], rel_l2=1e-2, what="block vs per-op")
-
-
 @pytest.mark.parametrize("recipe", ["paper", "unit_gate"])
 def test_tiny_fp32_step(recipe):
     wl = WL.standard_workloads()["tiny_fp32"]
@@ -332,24 +307,17 @@ def test_step_profile_matches_step_and_counts_launches():
         L = wl.n_layers
         assert kinds.count("attention") == L and kinds.count("attn_merge") == L
         assert kinds[-1] == "velocity"
-        if "block" in kinds:
-            # time embedding, 2 time-MLP layers, FiLM, embed+norm, layer-0 QKV; per
-            # layer attention, split merge (prefix 600 + 200 keys > 256) and the
-            # fused block (O, norm, gate/up, down, next norm + QKV or final norm);
-            # velocity
-            assert len(recs) == 6 + 3 * L + 1, kinds
-            assert kinds.count("block") == L and kinds.count("qkv") == 1
-        else:
-            # ... per layer QKV, attention, merge, O, norm, gate/up, down, norm (last
-            # layer: final norm); velocity
-            assert len(recs) == 5 + 8 * L + 1, kinds
-            assert kinds[-2] == "final_norm"
+        # time embedding, 2 time-MLP layers, FiLM, embed+norm; per layer QKV,
+        # attention, split merge (prefix 600 + 200 keys > 256), O-projection, norm,
+        # gate/up, down, norm (last layer: final norm); velocity
+        assert len(recs) == 5 + 8 * L + 1, kinds
+        assert kinds[-2] == "final_norm"
         assert all(us > 0 for _, _, us in recs)
     finally:
         case.close()
 
 
-def test_persistent_gemm_bitwise(monkeypatch):
+def test_persistent_gemm_bitwise():
     """The persistent projections (used where a projection has at least two
     output tiles per SM) give the per-operation kernels' results bit for bit:
     the same MMAs in the same order per tile, the same epilogues.  128 requests
@@ -357,14 +325,14 @@ def test_persistent_gemm_bitwise(monkeypatch):
     wl = WL.small_bf16_workload(batch=128, n_chunks=4, chunk_tokens=40, prefix_lens=[64] * 128)
     fresh = WL.make_fresh_noise(wl, 1)[0]
     results = {}
-    for mode in ("1", "0"):
-        monkeypatch.setenv("FVA_GEMM_PERSIST", mode)
-        case = Case(wl)
+    import paper_2608_27384_gb300 as fva
+    for mode, flags in (("persistent", 0), ("per_op", fva.FVA_FLAG_NO_PERSISTENT_GEMM)):
+        case = Case(wl, flags=flags)
         try:
             results[mode] = case.run(fresh=fresh)
         finally:
             case.close()
     for key in ("out", "buffer", "vel"):
-        a, b = results["1"][key], results["0"][key]
+        a, b = results["persistent"][key], results["per_op"][key]
         assert np.isfinite(a).all()
         assert np.array_equal(a.view(np.uint32), b.view(np.uint32)), key
