@@ -23,7 +23,14 @@
  *   - Device pointers are plain CUDA device addresses on the device that was
  *     current when fva_create ran; host pointers are ordinary host memory.
  *   - Asynchronous CUDA faults surface as FVA_ERR_CUDA from a later call.
- *   - A handle must not be used by two threads at once.
+ *   - A handle must not be used by two threads at once, nor on two streams whose
+ *     work can overlap: every queued call of a handle shares its parameter block,
+ *     workspaces and scratch, so the calls of one handle must be ordered on the
+ *     GPU (one stream per handle, or streams the caller orders with events).
+ *   - Every wait inside the library's kernels is bounded (2 s of GPU wall clock):
+ *     a kernel that gives up records a code in the handle's error word and
+ *     finishes without faulting; a later call returns FVA_ERR_TIMEOUT once (the
+ *     word is then cleared) and the calls after it run normally.
  */
 #ifndef FVA_H_
 #define FVA_H_
@@ -161,6 +168,24 @@ fva_status fva_set_prefix_kv(fva_handle* h, int32_t request, int32_t layer, cons
                              const void* v, int32_t len, int32_t on_device, fva_stream stream);
 
 /*
+ * Let `request` use the prefix K/V of `src_request` (every layer, same length)
+ * without a copy of it: the attention reads the shared prefix keys and values from
+ * src_request's rows.  Only the prefix rows past the last multiple of 64 (fewer than
+ * 64 per layer; the whole prefix on an fp32 handle is still read from the source)
+ * are copied into request's rows, because the attention's 64-key block that
+ * straddles the prefix end also holds request's own action keys.  This is the
+ * packed multi-buffer forward of the paper (§3.3, App. A.4): N buffer
+ * configurations of one observation, separated by the mask and reading one prefix.
+ * The share lasts until either request's prefix is set again: setting
+ * src_request's prefix (fva_set_prefix_kv) drops the share, and request's next
+ * step then returns FVA_ERR_STATE until it is set or shared again.  Queued on
+ * `stream`.  Errors: INVALID_ARG (request out of range or equal to src_request),
+ * STATE (src_request has no complete prefix, or itself shares one), CUDA.
+ */
+fva_status fva_share_prefix_kv(fva_handle* h, int32_t request, int32_t src_request,
+                               fva_stream stream);
+
+/*
  * One steady-streaming step (§3.2, Algorithm 1; Eq. 1 and 2) for `batch`
  * independent requests, queued on `stream`; returns without waiting.
  *   buffer       device fp32 [batch, K, H, A], slot 0 = cleanest chunk; updated in
@@ -246,10 +271,20 @@ fva_status fva_mask_table(fva_handle* h, int32_t batch, int32_t* key_limit, fva_
  * softmax scale 1/sqrt(head_dim).  Uses the handle's split-KV scratch, so calls
  * on one handle must not overlap on the GPU.  Requires 1 <= batch <= max_batch and
  * kv_rows <= max_prefix + K*H, and 16-byte aligned pointers.  Errors: INVALID_ARG,
- * UNSUPPORTED (fp32 handle), CUDA.  A device P_r that breaks P_r + K*H <= kv_rows
- * cannot be seen on the host: the kernel leaves those rows unwritten and the
- * next fva_step on the handle returns FVA_ERR_INVALID_ARG.
+ * UNSUPPORTED (fp32 handle), CUDA.  A device P_r that breaks 0 <= P_r and
+ * P_r + K*H <= kv_rows cannot be seen on the host: the kernel leaves request r's
+ * rows unwritten and the next fva_step on the handle returns FVA_ERR_INVALID_ARG.
  */
+
+/*
+ * The tanh-form GELU exactly as the bf16 gate/up epilogue evaluates it, before the
+ * product with the up branch and the bf16 rounding (the fp32 dtype uses a separate,
+ * full-precision form): y[i] = 0.5 x (1 + tanh(sqrt(2/pi) (x + 0.044715 x^3))) with
+ * tanh from the PTX tanh.approx.f32 instruction, whose absolute error bound makes
+ * |y - GELU(x)| <= |x| 2^-12.  x and y are device fp32 arrays of n >= 0 elements.
+ * Errors: INVALID_ARG, CUDA.
+ */
+fva_status fva_geglu_gelu(const float* x, float* y, int64_t n, fva_stream stream);
 fva_status fva_chunk_attention(fva_handle* h, const void* q, const void* k, const void* v,
                                const int32_t* prefix_len, int32_t batch, int32_t kv_rows,
                                void* out, fva_stream stream);
@@ -261,8 +296,10 @@ fva_status fva_chunk_attention(fva_handle* h, const void* q, const void* k, cons
  * cudaMalloc / cudaFree may synchronise the device for an unbounded time, or a
  * host that gives all device memory to its own pool at start-up.
  *
- * Same inputs, output and numerics as fva_chunk_attention, with the shapes passed
- * explicitly (head_dim must be 256, n_q_heads one of 1, 2, 4, 8, 16).  The split-KV
+ * Same inputs, output, kernel and mask as fva_chunk_attention, with the shapes
+ * passed explicitly (head_dim must be 256, n_q_heads one of 1, 2, 4, 8, 16).  Its
+ * key splits are always 256 keys, while a handle may use shorter ones, so the two
+ * can differ by bf16 rounding.  The split-KV
  * scratch is a fixed array inside the library: 256 slots of 128 x 256 bf16 plus
  * row statistics (16 MiB + 256 KiB), kept by every GPU that loads the library
  * until the process exits.  A call needs
@@ -272,8 +309,9 @@ fva_status fva_chunk_attention(fva_handle* h, const void* q, const void* k, cons
  * kernel attributes) with that device current; make that first call before any
  * stream capture.  Every call uses the same array, which keeps the last call's
  * contents (nothing in it needs to start at zero): calls that overlap on the GPU,
- * from any thread or stream, race.  Device-side problems (a prefix length beyond
- * kv_rows - K*H) leave the affected rows unwritten and are not reported.
+ * from any thread or stream, race.  Device-side problems (a prefix length P_r with
+ * P_r + K*H > kv_rows, or P_r < 0) leave request r's rows unwritten and are not
+ * reported.
  * Calls no cudaMalloc, cudaFree or other allocating routine.
  */
 fva_status fva_chunk_attention_noalloc(const void* q, const void* k, const void* v,
@@ -281,6 +319,17 @@ fva_status fva_chunk_attention_noalloc(const void* q, const void* k, const void*
                                        int32_t n_chunks, int32_t chunk_tokens,
                                        int32_t n_q_heads, int32_t head_dim, int32_t kv_rows,
                                        void* out, fva_stream stream);
+
+/*
+ * Test hook of the bounded waits (no counterpart in the paper).  Queues on
+ * `stream` one kernel whose only wait can never complete: after limit_us
+ * (1 .. 1000000) microseconds of GPU wall clock it records a timeout code in the
+ * handle's error word and returns, as every bounded wait of the library does.
+ * The first fva_step / fva_step_ex issued after the stream has passed that point
+ * (e.g. after synchronising it) returns FVA_ERR_TIMEOUT without queuing work;
+ * the step after that runs normally.  Errors: INVALID_ARG, CUDA.
+ */
+fva_status fva_check_bounded_wait(fva_handle* h, int32_t limit_us, fva_stream stream);
 
 /* Kernels of one step, as reported by fva_step_profile. */
 typedef enum fva_kernel_kind {

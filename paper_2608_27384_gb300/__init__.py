@@ -68,6 +68,7 @@ EXPORTS = ["fva_create", "fva_destroy", "fva_num_weights", "fva_weight_shape",
            "fva_load_weights", "fva_set_prefix_kv", "fva_step", "fva_step_ex",
            "fva_trace_floats", "fva_set_step_index", "fva_get_step_index", "fva_mask_table",
            "fva_step_profile", "fva_chunk_attention", "fva_chunk_attention_noalloc",
+           "fva_check_bounded_wait", "fva_geglu_gelu", "fva_share_prefix_kv",
            "fva_last_error"]
 
 _lib_handle: Optional[ctypes.CDLL] = None
@@ -97,6 +98,9 @@ def lib() -> ctypes.CDLL:
         "fva_set_step_index": (i32, [vp, u64]),
         "fva_get_step_index": (i32, [vp, P(u64)]),
         "fva_mask_table": (i32, [vp, i32, vp, vp]),
+        "fva_check_bounded_wait": (i32, [vp, i32, vp]),
+        "fva_share_prefix_kv": (i32, [vp, i32, i32, vp]),
+        "fva_geglu_gelu": (i32, [vp, vp, ctypes.c_int64, vp]),
         "fva_step_profile": (i32, [vp, vp, P(ctypes.c_float), vp, i32, P(fva_kernel_time), i32,
                                    P(i32), vp]),
         "fva_chunk_attention": (i32, [vp, vp, vp, vp, vp, i32, i32, vp, vp]),
@@ -224,6 +228,18 @@ def fva_get_step_index(handle: int) -> int:
 
 def fva_mask_table(handle: int, batch: int, key_limit, stream=None) -> None:
     _check(lib().fva_mask_table(handle, batch, _ptr(key_limit), _stream(stream)))
+
+
+def fva_share_prefix_kv(handle: int, request: int, src_request: int, stream=None) -> None:
+    _check(lib().fva_share_prefix_kv(handle, request, src_request, _stream(stream)))
+
+
+def fva_geglu_gelu(x, y, n: int, stream=None) -> None:
+    _check(lib().fva_geglu_gelu(_ptr(x), _ptr(y), n, _stream(stream)))
+
+
+def fva_check_bounded_wait(handle: int, limit_us: int, stream=None) -> None:
+    _check(lib().fva_check_bounded_wait(handle, limit_us, _stream(stream)))
 
 
 def fva_step_profile(handle: int, buffer, noise_levels, out_chunk, batch: int, stream=None):

@@ -9,9 +9,9 @@
 // no allocating routine: the attention's split-KV scratch lives in a fixed
 // file-scope device array instead.
 //
-// The array is kNoAllocSlots partial tiles (128 rows x 256 fp32 each, plus their
-// row max / sum): 32 MiB + 256 KiB, held by every GPU that loads libfva until the
-// process exits.  A call needs batch * ceil(K*H*nq / 128) * ceil(kv_rows / 256)
+// The array is kNoAllocSlots partial tiles (128 rows x 256 bf16 each, plus their
+// row max / sum as fp32 pairs): 16 MiB + 256 KiB, held by every GPU that loads
+// libfva until the process exits.  A call needs batch * ceil(K*H*nq / 128) * ceil(kv_rows / 256)
 // slots; larger calls are rejected.
 #include <cudaTypedefs.h>
 

@@ -92,19 +92,25 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Wait for the phase with the given parity to complete.  Gives up after
-// kWaitLimitNs, records `code` in *err and returns false.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err, int code) {
+// Wait for the phase with the given parity to complete.  Gives up after limit_ns
+// of %globaltimer, records `code` in *err and returns false.
+__device__ __forceinline__ bool mbar_wait_ns(uint64_t* bar, uint32_t parity, int* err, int code,
+                                             unsigned long long limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer_ns();
   uint32_t n = 0;
   while (!mbar_try_wait(bar, parity)) {
-    if ((++n & 255u) == 0u && globaltimer_ns() - t0 > kWaitLimitNs) {
+    if ((++n & 255u) == 0 && globaltimer_ns() - t0 > limit_ns) {
       report_error(err, code);
       return false;
     }
   }
   return true;
+}
+
+// The same with the library's limit, kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err, int code) {
+  return mbar_wait_ns(bar, parity, err, code, kWaitLimitNs);
 }
 
 // ----------------------------------------------------------------------------
@@ -331,7 +337,9 @@ __device__ __forceinline__ float gelu_tanh_f(float x) {
 
 // The same GELU for bf16 outputs: tanh(u) by the PTX tanh.approx.f32 instruction
 // (one special-function operation instead of two).  Its absolute error of about
-// 2^-11 leaves an absolute error of at most |x| 2^-12 in the result.
+// 2^-11 leaves an absolute error of at most |x| 2^-12 in the result (checked on the
+// GPU through fva_geglu_gelu).  Only for results rounded to bf16: the fp32 path
+// uses gelu_tanh_f.
 __device__ __forceinline__ float gelu_tanh_bf16out(float x) {
   const float k0 = 0.7978845608028654f;  // sqrt(2 / pi)
   const float u = k0 * fmaf(0.044715f * x, x * x, x);

@@ -146,6 +146,8 @@ struct fva_handle {
   // prefix / KV workspace
   void *kc = nullptr, *vc = nullptr;
   int* prefix_len_dev = nullptr;
+  int* prefix_src_dev = nullptr;  // [Bmax]: request whose rows hold the prefix keys
+  std::vector<int> prefix_src;    // host copy
   std::vector<int> layer_len;  // [Bmax * L], -1 = never set
   float2* rope = nullptr;
   uint32_t* rope_h = nullptr;  // fp16 copy for the bf16 QKV epilogue
@@ -347,6 +349,8 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
   h->Mmax = h->Bmax * h->T;
   h->layers.resize(h->L);
   h->layer_len.assign((size_t)h->Bmax * h->L, -1);
+  h->prefix_src.resize(h->Bmax);
+  for (int r = 0; r < h->Bmax; ++r) h->prefix_src[r] = r;
   CUDA_TRY(cudaGetDevice(&h->device));
   fva_status st;
   if (h->bf16) {
@@ -361,6 +365,7 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
   const size_t kv_elems = (size_t)h->L * h->Bmax * h->S_cap * h->dh;
   if ((st = dalloc(h, &h->kc, kv_elems, a)) || (st = dalloc(h, &h->vc, kv_elems, a)) ||
       (st = dalloc(h, &h->prefix_len_dev, h->Bmax)) ||
+      (st = dalloc(h, &h->prefix_src_dev, h->Bmax)) ||
       (st = dalloc(h, &h->rope, (size_t)h->S_cap * (h->dh / 2))) ||
       (st = dalloc(h, &h->rope_h, (size_t)h->S_cap * (h->dh / 2))) ||
       (st = dalloc(h, &h->temb, (size_t)h->BKmax * h->W, a)) ||
@@ -723,6 +728,23 @@ extern "C" fva_status fva_load_weights(fva_handle* h, const void* const* tensors
 // =============================================================================
 namespace {
 __global__ void set_len_kernel(int* dst, int v) { *dst = v; }
+__global__ void set_share_kernel(int* len, int* src, int r, int v, int s) {
+  len[r] = v;
+  src[r] = s;
+}
+
+// Request r's prefix was replaced: requests that shared it lose the share (their
+// steps report a missing prefix until they are set or shared again), and r itself
+// reads its own rows again.
+void drop_shares_of(fva_handle* h, int r, cudaStream_t s) {
+  for (int q = 0; q < h->Bmax; ++q)
+    if (q != r && h->prefix_src[q] == r) {
+      h->prefix_src[q] = q;
+      for (int l = 0; l < h->L; ++l) h->layer_len[(size_t)q * h->L + l] = -1;
+      set_share_kernel<<<1, 1, 0, s>>>(h->prefix_len_dev, h->prefix_src_dev, q, 0, q);
+    }
+  h->prefix_src[r] = r;
+}
 }  // namespace
 
 extern "C" fva_status fva_set_prefix_kv(fva_handle* h, int32_t request, int32_t layer,
@@ -738,6 +760,7 @@ extern "C" fva_status fva_set_prefix_kv(fva_handle* h, int32_t request, int32_t 
   if (len > 0 && (!k || !v)) return fail(FVA_ERR_INVALID_ARG, "k or v is NULL");
   DeviceGuard guard(h->device);
   cudaStream_t s = (cudaStream_t)stream;
+  drop_shares_of(h, request, s);
   const size_t row = (size_t)h->dh * h->act, bytes = (size_t)len * row;
   const cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
   const int l0 = layer < 0 ? 0 : layer, l1 = layer < 0 ? h->L : layer + 1;
@@ -750,7 +773,45 @@ extern "C" fva_status fva_set_prefix_kv(fva_handle* h, int32_t request, int32_t 
     }
     h->layer_len[(size_t)request * h->L + l] = len;
   }
-  set_len_kernel<<<1, 1, 0, s>>>(h->prefix_len_dev + request, len);
+  set_share_kernel<<<1, 1, 0, s>>>(h->prefix_len_dev, h->prefix_src_dev, request, len, request);
+  CUDA_TRY(cudaGetLastError());
+  return FVA_OK;
+}
+
+extern "C" fva_status fva_share_prefix_kv(fva_handle* h, int32_t request, int32_t src_request,
+                                          fva_stream stream) {
+  if (!h) return fail(FVA_ERR_INVALID_ARG, "handle is NULL");
+  if (request < 0 || request >= h->Bmax || src_request < 0 || src_request >= h->Bmax)
+    return fail(FVA_ERR_INVALID_ARG, "request %d / src_request %d outside [0, %d)", request,
+                src_request, h->Bmax);
+  if (request == src_request) return fail(FVA_ERR_INVALID_ARG, "a request cannot share itself");
+  if (h->prefix_src[src_request] != src_request)
+    return fail(FVA_ERR_STATE, "request %d itself shares another request's prefix", src_request);
+  const int len = h->layer_len[(size_t)src_request * h->L];
+  for (int l = 0; l < h->L; ++l)
+    if (len < 0 || h->layer_len[(size_t)src_request * h->L + l] != len)
+      return fail(FVA_ERR_STATE, "request %d has no complete prefix K/V", src_request);
+  DeviceGuard guard(h->device);
+  cudaStream_t s = (cudaStream_t)stream;
+  drop_shares_of(h, request, s);
+  // the 64-key block that straddles the prefix end also holds action keys, so it
+  // is read from this request's rows: copy the prefix tail there
+  const int tail0 = h->bf16 ? (len / 64) * 64 : len;
+  const size_t row = (size_t)h->dh * h->act;
+  for (int l = 0; l < h->L; ++l) {
+    const size_t src = (((size_t)l * h->Bmax + src_request) * h->S_cap + tail0) * row;
+    const size_t dst = (((size_t)l * h->Bmax + request) * h->S_cap + tail0) * row;
+    if (len > tail0) {
+      CUDA_TRY(cudaMemcpyAsync((uint8_t*)h->kc + dst, (const uint8_t*)h->kc + src,
+                               (size_t)(len - tail0) * row, cudaMemcpyDeviceToDevice, s));
+      CUDA_TRY(cudaMemcpyAsync((uint8_t*)h->vc + dst, (const uint8_t*)h->vc + src,
+                               (size_t)(len - tail0) * row, cudaMemcpyDeviceToDevice, s));
+    }
+    h->layer_len[(size_t)request * h->L + l] = len;
+  }
+  h->prefix_src[request] = src_request;
+  set_share_kernel<<<1, 1, 0, s>>>(h->prefix_len_dev, h->prefix_src_dev, request, len,
+                                   src_request);
   CUDA_TRY(cudaGetLastError());
   return FVA_OK;
 }
@@ -950,6 +1011,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       aa.err = h->err_dev;
       aa.pad_tokens = h->pad_dev();
       aa.block_diag = (h->cfg.flags & FVA_FLAG_BLOCK_DIAGONAL) ? 1 : 0;
+      aa.prefix_src = h->prefix_src_dev;
       mark(FVA_K_ATTENTION, l);
       CUDA_TRY(launch_tc_attention(&h->m_q, &h->m_k, &h->m_v, aa, B, s));
       if (aa.max_splits > 1) {
@@ -959,7 +1021,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     } else {
       launch_f32_attention((float*)h->q, (float*)kc_l, (float*)vc_l, h->prefix_len_dev,
                            h->pad_dev(), (h->cfg.flags & FVA_FLAG_BLOCK_DIAGONAL) ? 1 : 0,
-                           (float*)h->attn, B, h->T, h->H, h->nq, h->dh, h->S_cap, h->S_cap, s);
+                           h->prefix_src_dev, (float*)h->attn, B, h->T, h->H, h->nq, h->dh, h->S_cap, h->S_cap, s);
     }
     if (trace) launch_to_f32(h->attn, bf, tr_at(o_att), (long long)M * Dq, s);
     // output projection (split-K partials) -> gated residual + norm 2
@@ -1023,10 +1085,16 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   return FVA_OK;
 }
 
-fva_status check_async_error(fva_handle* h) {
+// Reports the device error word once it has been read back, and clears it so that
+// the calls after the reported one run normally.  `s` is the calling step's stream.
+fva_status check_async_error(fva_handle* h, cudaStream_t s) {
   if (h->err_pending && cudaEventQuery(h->err_ev) == cudaSuccess) {
     h->err_pending = false;
     const int code = *h->err_host;
+    if (code != 0) {
+      *h->err_host = 0;
+      CUDA_TRY(cudaMemsetAsync(h->err_dev, 0, sizeof(int), s));
+    }
     if (code == 4 /* KERR_BAD_SHAPE */)
       return fail(FVA_ERR_INVALID_ARG, "an earlier kernel saw a device size beyond its bound");
     if (code != 0)
@@ -1121,9 +1189,9 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     }
   }
   DeviceGuard guard(h->device);
-  fva_status st = check_async_error(h);
-  if (st != FVA_OK) return st;
   cudaStream_t s = (cudaStream_t)stream;
+  fva_status st = check_async_error(h, s);
+  if (st != FVA_OK) return st;
 
   // stage tau, dt and the step index through a pinned ring slot
   const int slot = h->ring_pos;
@@ -1264,6 +1332,46 @@ extern "C" fva_status fva_mask_table(fva_handle* h, int32_t batch, int32_t* key_
   DeviceGuard guard(h->device);
   launch_mask_table(h->prefix_len_dev, batch, h->T, h->H, key_limit, (cudaStream_t)stream);
   CUDA_TRY(cudaGetLastError());
+  return FVA_OK;
+}
+
+extern "C" fva_status fva_geglu_gelu(const float* x, float* y, int64_t n, fva_stream stream) {
+  if (n < 0 || (n > 0 && (!x || !y))) return fail(FVA_ERR_INVALID_ARG, "bad x / y / n");
+  launch_geglu_gelu(x, y, n, (cudaStream_t)stream);
+  CUDA_TRY(cudaGetLastError());
+  return FVA_OK;
+}
+
+// =============================================================================
+// bounded-wait check
+// =============================================================================
+namespace {
+// One thread waits on an mbarrier that nothing arrives at, with a wall-clock limit
+// of limit_ns: when the limit passes it records KERR_WAIT_SYNC in *err and returns,
+// the same path every bounded wait of the library's kernels takes.
+__global__ void stall_kernel(int* err, unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  fence_barrier_init();
+  mbar_wait_ns(&bar, 0, err, KERR_WAIT_SYNC, limit_ns);
+}
+}  // namespace
+
+extern "C" fva_status fva_check_bounded_wait(fva_handle* h, int32_t limit_us, fva_stream stream) {
+  if (!h) return fail(FVA_ERR_INVALID_ARG, "handle is NULL");
+  if (limit_us < 1 || limit_us > 1000000)
+    return fail(FVA_ERR_INVALID_ARG, "limit_us %d outside [1, 1000000]", limit_us);
+  DeviceGuard guard(h->device);
+  cudaStream_t s = (cudaStream_t)stream;
+  stall_kernel<<<1, 32, 0, s>>>(h->err_dev, (unsigned long long)limit_us * 1000ull);
+  CUDA_TRY(cudaGetLastError());
+  // read the error word back behind it (replacing any read-back still pending: this
+  // one also sees what an earlier one would), so the next call reports it once the
+  // stream has passed this point
+  CUDA_TRY(cudaMemcpyAsync(h->err_host, h->err_dev, sizeof(int), cudaMemcpyDeviceToHost, s));
+  CUDA_TRY(cudaEventRecord(h->err_ev, s));
+  h->err_pending = true;
   return FVA_OK;
 }
 

@@ -86,6 +86,9 @@ void launch_gather_action_kv(const void* kv_layer, bool act_bf16, const int* pre
 void launch_mask_table(const int* prefix_len, int B, int T, int H, int* key_limit,
                        cudaStream_t s);
 
+// y = the bf16 GeGLU epilogue's GELU of x (fp32 in and out).
+void launch_geglu_gelu(const float* x, float* y, long long n, cudaStream_t s);
+
 
 // ---------------------------------------------------------------- tc_gemm.cu
 enum GemmMode {
@@ -160,6 +163,9 @@ struct AttnArgs {
   // own chunk start.
   const int* pad_tokens;
   int block_diag;
+  // Key blocks wholly inside request r's prefix are read from the KV rows of
+  // request prefix_src[r] (a shared prefix); nullptr: every request its own.
+  const int* prefix_src;
 };
 
 constexpr int kAttnKeysPerSplit = 256;
@@ -183,9 +189,11 @@ void launch_f32_qkv_rope(const float* C, float* q, float* kc, float* vc,
                          const int* prefix_len, const float2* rope, int M, int T, int S_cap,
                          int nq, int dh, cudaStream_t s);
 void launch_f32_geglu(const float* C, float* out, int M, int F, cudaStream_t s);
+// prefix_src: per request, the request whose KV rows hold its prefix keys
+// (nullptr: its own).
 void launch_f32_attention(const float* q, const float* kc, const float* vc,
                           const int* prefix_len, const int* pad_tokens, int block_diag,
-                          float* out, int B, int T, int H, int nq, int dh, int S_cap,
-                          int max_keys, cudaStream_t s);
+                          const int* prefix_src, float* out, int B, int T, int H, int nq, int dh,
+                          int S_cap, int max_keys, cudaStream_t s);
 
 }  // namespace fva

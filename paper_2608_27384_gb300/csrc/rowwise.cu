@@ -3,6 +3,8 @@
 // residual + FiLM RMSNorm, and the fused final norm + out-projection + Euler
 // update + emit + buffer roll + tail noise.  Plus small table / debug helpers.
 #include <cuda_fp16.h>
+
+#include <algorithm>
 #include "common.cuh"
 #include "kernels.h"
 
@@ -697,6 +699,19 @@ void launch_gemv_silu(const void* in, const void* w, const float* bias, void* ou
   launch_pdl(gemv_silu_kernel, dim3((N + kGemvWarps - 1) / kGemvWarps), dim3(32 * kGemvWarps),
              (size_t)kGemvRows * K * 2, s, (const bf16*)in, (const bf16*)w, bias, (bf16*)out, M, N,
              K);
+}
+
+// The bf16 GeGLU epilogue's GELU on an fp32 array (introspection of its accuracy).
+__global__ void geglu_gelu_kernel(const float* __restrict__ x, float* __restrict__ y, long long n) {
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n;
+       i += (long long)gridDim.x * blockDim.x)
+    y[i] = gelu_tanh_bf16out(x[i]);
+}
+
+void launch_geglu_gelu(const float* x, float* y, long long n, cudaStream_t s) {
+  if (n <= 0) return;
+  const long long blocks = std::min<long long>((n + 255) / 256, 4096);
+  geglu_gelu_kernel<<<(unsigned)blocks, 256, 0, s>>>(x, y, n);
 }
 
 // ----------------------------------------------------------------------------

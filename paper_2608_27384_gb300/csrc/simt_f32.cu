@@ -134,6 +134,7 @@ __global__ void f32_attention_kernel(const float* __restrict__ q, const float* _
                                      const float* __restrict__ vc,
                                      const int* __restrict__ prefix_len,
                                      const int* __restrict__ pad_tokens, int block_diag,
+                                     const int* __restrict__ prefix_src,
                                      float* __restrict__ out, int T, int H, int nq, int dh,
                                      int S_cap) {
   extern __shared__ float sm[];  // [dh] query, then [limit] scores
@@ -154,9 +155,14 @@ __global__ void f32_attention_kernel(const float* __restrict__ q, const float* _
   const float scale = rsqrtf((float)dh);
   const float* K = kc + (size_t)r * S_cap * dh;
   const float* V = vc + (size_t)r * S_cap * dh;
+  // a request that shares another's prefix reads the prefix keys from its rows
+  const int src = prefix_src ? prefix_src[r] : r;
+  const float* Ks = kc + (size_t)src * S_cap * dh;
+  const float* Vs = vc + (size_t)src * S_cap * dh;
   for (int s = threadIdx.x; s < limit; s += blockDim.x) {
+    const float* krow = (s < P ? Ks : K) + (size_t)s * dh;
     float acc = 0.f;
-    for (int d = 0; d < dh; ++d) acc = fmaf(sq[d], K[(size_t)s * dh + d], acc);
+    for (int d = 0; d < dh; ++d) acc = fmaf(sq[d], krow[d], acc);
     sc[s] = (s < P || s >= lo) ? acc * scale : -INFINITY;
   }
   __syncthreads();
@@ -184,20 +190,20 @@ __global__ void f32_attention_kernel(const float* __restrict__ q, const float* _
   float* orow = out + ((size_t)m * nq + head) * dh;
   for (int d = threadIdx.x; d < dh; d += blockDim.x) {
     float acc = 0.f;
-    for (int s = 0; s < limit; ++s) acc = fmaf(sc[s], V[(size_t)s * dh + d], acc);
+    for (int s = 0; s < limit; ++s) acc = fmaf(sc[s], (s < P ? Vs : V)[(size_t)s * dh + d], acc);
     orow[d] = acc * inv;
   }
 }
 
 void launch_f32_attention(const float* q, const float* kc, const float* vc,
                           const int* prefix_len, const int* pad_tokens, int block_diag,
-                          float* out, int B, int T, int H, int nq, int dh, int S_cap,
-                          int max_keys, cudaStream_t s) {
+                          const int* prefix_src, float* out, int B, int T, int H, int nq, int dh,
+                          int S_cap, int max_keys, cudaStream_t s) {
   if (B * T <= 0) return;
   dim3 grid(B * T, nq);
   const size_t smem = sizeof(float) * (dh + max_keys);
   launch_pdl(f32_attention_kernel, grid, dim3(128), smem, s, q, kc, vc, prefix_len, pad_tokens,
-             block_diag, out, T, H, nq, dh, S_cap);
+             block_diag, prefix_src, out, T, H, nq, dh, S_cap);
 }
 
 }  // namespace fva

@@ -119,6 +119,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int qrow0 = (r * a.T + t0) * a.nq;
   const int krow0 = a.kv_row0 + r * a.S_cap + kb0 * kKB;
+  // blocks wholly inside the prefix of a request that shares another's prefix come
+  // from that request's rows (same keys; the block that straddles P comes from this
+  // request's own rows, which hold its copy of the prefix tail)
+  const int src = a.prefix_src ? __ldg(a.prefix_src + r) : r;
+  const int krow0_src = a.kv_row0 + src * a.S_cap + kb0 * kKB;
 
   if (warp == 0 && lane == 0) {
     // ---------------- TMA producer
@@ -129,9 +134,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     // while later slabs are in flight.  Every other thread only runs behind
     // these loads.
     constexpr uint32_t kSlab = kBlocksPerSplit * kKB * 128;
+    auto row_of = [&](int b) {
+      return ((kb0 + b + 1) * kKB <= P ? krow0_src : krow0) + b * kKB;
+    };
     auto load_k = [&](int j, int b) {
       mbar_arrive_expect_tx(&qk_full[j], kKB * 128);
-      tma_load_2d(sKV + j * kSlab + b * (kKB * 128), &tmK, j * 64, krow0 + b * kKB, &qk_full[j]);
+      tma_load_2d(sKV + j * kSlab + b * (kKB * 128), &tmK, j * 64, row_of(b), &qk_full[j]);
     };
     int npre = 0;
     while (npre < nblk && (kb0 + npre + 1) * kKB <= P) ++npre;
@@ -147,8 +155,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int b = 0; b < nblk; ++b) {
         mbar_arrive_expect_tx(&v_full[b], kKVBytes);
         for (int j = 0; j < 4; ++j)
-          tma_load_2d(sKV + j * kSlab + b * (kKB * 128), &tmV, j * 64, krow0 + b * kKB,
-                      &v_full[b]);
+          tma_load_2d(sKV + j * kSlab + b * (kKB * 128), &tmV, j * 64, row_of(b), &v_full[b]);
       }
   } else if (warp == 1 && lane == 0) {
     // ---------------- MMA issuer

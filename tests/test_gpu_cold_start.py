@@ -144,18 +144,19 @@ def test_block_diagonal_mask(dtype):
 def test_multi_buffer_forward():
     """The packed multi-buffer forward (§3.3, App. A.4): the N cold-start
     configurations of one observation, [pad x (N-j), j real chunks] for j = 1..N,
-    sharing one prefix and isolated from each other, in one launch as a batch of
-    N requests.  Each configuration matches the oracle, and equals running it
-    alone bit for bit (no cross-buffer interaction)."""
+    reading one shared prefix K/V (fva_share_prefix_kv) and isolated from each
+    other, in one launch as a batch of N requests.  Each configuration matches the
+    oracle, and equals running it alone bit for bit (no cross-buffer interaction)."""
     K = 3
     base = _workload("bf16", n_chunks=K)
     wl = WL.Workload(**dict(base.__dict__, batch=K, prefix_lens=[base.prefix_lens[0]] * K))
     case = Case(wl)
     try:
+        import paper_2608_27384_gb300 as fva
         buf = np.repeat(case.buf[:1], K, axis=0)              # the same future chunks...
-        pre = [case.prefix[0]] * K                            # ...and the same observation
-        for r in range(K):
-            case.dec.set_prefix(r, pre[r][0], pre[r][1])
+        pre = [case.prefix[0]] * K                            # ...and the same observation,
+        for r in range(1, K):                                 # read from request 0's rows
+            fva.fva_share_prefix_kv(case.handle, r, 0)
         case.prefix = pre
         n_valid = list(range(1, K + 1))
         fresh = WL.make_fresh_noise(wl, 1)[0]
@@ -165,5 +166,45 @@ def test_multi_buffer_forward():
             alone = case.run(buf=buf[r:r + 1], fresh=fresh[r:r + 1], n_valid=[n_valid[r]], batch=1)
             c0 = K - n_valid[r]
             np.testing.assert_array_equal(res["vel"][r, c0:], alone["vel"][0, c0:])
+    finally:
+        case.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_shared_prefix_equals_separate_copies(dtype):
+    """A request reading another's prefix (fva_share_prefix_kv) gives the same
+    results bit for bit as the same prefix uploaded into its own rows; setting the
+    source's prefix again drops the share."""
+    import paper_2608_27384_gb300 as fva
+    base = _workload(dtype, n_chunks=3)
+    P = 150 if dtype == "bf16" else base.prefix_lens[0]  # 150 = 2 x 64 + a 22-key tail
+    wl = WL.Workload(**dict(base.__dict__, batch=3, prefix_lens=[P] * 3))
+    case = Case(wl)
+    try:
+        buf = case.buf
+        fresh = WL.make_fresh_noise(wl, 1)[0]
+        for r in range(3):                           # separate copies of request 0's prefix
+            case.dec.set_prefix(r, case.prefix[0][0], case.prefix[0][1])
+        sep = case.run(buf=buf, fresh=fresh)
+        for r in (1, 2):                             # the same prefix, shared
+            fva.fva_share_prefix_kv(case.handle, r, 0)
+        shr = case.run(buf=buf, fresh=fresh)
+        for key in ("out", "buffer", "vel"):
+            np.testing.assert_array_equal(sep[key], shr[key])
+        case.prefix = [case.prefix[0]] * 3
+        out_ref, new_ref, _ = case.oracle_step(buf=buf, fresh=fresh)
+        tol = TOL[dtype]
+        assert_close(shr["out"], out_ref, what="shared out", **tol)
+        assert_close(shr["buffer"], new_ref, what="shared buffer", **tol)
+        with pytest.raises(fva.FvaError) as e:
+            fva.fva_share_prefix_kv(case.handle, 1, 1)
+        assert e.value.name == "FVA_ERR_INVALID_ARG"
+        with pytest.raises(fva.FvaError) as e:
+            fva.fva_share_prefix_kv(case.handle, 0, 1)    # 1 itself shares 0's prefix
+        assert e.value.name == "FVA_ERR_STATE"
+        case.dec.set_prefix(0, case.prefix[0][0], case.prefix[0][1])  # drops the shares
+        with pytest.raises(fva.FvaError) as e:
+            case.run(buf=buf, fresh=fresh)
+        assert e.value.name == "FVA_ERR_STATE"
     finally:
         case.close()

@@ -11,7 +11,7 @@ import numpy as np
 import pytest
 
 from gpu_util import assert_close
-from test_gpu_attention import attention_inputs, make_handle
+from test_gpu_attention import attention_inputs, make_handle, oracle_attention
 
 pytestmark = pytest.mark.gpu
 
@@ -38,7 +38,8 @@ def test_noalloc_matches_allocating_entry_point_twice_in_a_row():
     import torch
     import paper_2608_27384_gb300 as fva
     # two different calls back to back: the fixed scratch keeps the first call's
-    # partials, which the second must not pick up
+    # partials, which the second must not pick up.  Slots used: 32 tiles x 5 splits =
+    # 160, then 2 requests x 32 tiles x 4 splits = 256, exactly the array's 256 slots.
     cases = [([560], 10, 50, 8, 1), ([300, 200], 10, 50, 8, 2)]
     for prefix_lens, K, H, nq, seed in cases:
         q, k, v, kv_rows = attention_inputs(prefix_lens, K, H, nq, seed=seed)
@@ -58,6 +59,30 @@ def test_noalloc_matches_allocating_entry_point_twice_in_a_row():
         got, ref = _to_f32(out_new), _to_f32(out_ref)
         assert np.all(np.isfinite(got))
         assert_close(got, ref, max_abs=2e-2, rel_l2=1e-2, what=f"noalloc P={prefix_lens}")
+
+
+@pytest.mark.parametrize("prefix_lens,K,H,nq", [
+    # slots = batch * ceil(K*H*nq / 128) * ceil(kv_rows / 256)
+    ([129], 3, 50, 4),           # 5 tiles x 2 splits = 10 slots
+    ([300, 45], 2, 50, 16),      # 2 requests x 13 tiles x 2 splits = 52 slots
+    ([560], 10, 50, 8),          # 32 tiles x 5 splits = 160 slots
+])
+def test_noalloc_matches_oracle(prefix_lens, K, H, nq):
+    """The no-allocation entry point against the fp64 oracle directly, for several
+    query-head counts (each changes the tokens per 128-row tile and the tile count)."""
+    import torch
+    import paper_2608_27384_gb300 as fva
+    q, k, v, kv_rows = attention_inputs(prefix_lens, K, H, nq, seed=3)
+    B = len(prefix_lens)
+    dq, dk, dv = _dev_bits(q), _dev_bits(k), _dev_bits(v)
+    dp = torch.tensor(prefix_lens, dtype=torch.int32, device="cuda")
+    out = torch.full_like(dq, -1)
+    for _ in range(2):  # twice in a row: the shared scratch keeps the last call's data
+        fva.fva_chunk_attention_noalloc(dq, dk, dv, dp, B, K, H, nq, 256, kv_rows, out)
+        torch.cuda.synchronize()
+        got = _to_f32(out)
+        ref = oracle_attention(q, k, v, prefix_lens, K, H, nq)
+        assert_close(got, ref, max_abs=2e-2, rel_l2=1e-2, what=f"noalloc vs oracle nq={nq}")
 
 
 def test_noalloc_rejects_calls_beyond_its_fixed_scratch():
