@@ -122,16 +122,20 @@ def kernel_costs(wl, B, n_sms=152):
     return c
 
 
-def step_costs(wl, B):
+def step_costs(wl, B, film=True):
     """Whole-step algorithmic FLOPs and the HBM bytes that must be streamed (every
-    weight once + the prefix K/V of every layer)."""
+    weight once + the prefix K/V of every layer).  film=False: the step that reuses
+    the previous step's FiLM modulation (no time MLP, no FiLM projection)."""
     L = wl.n_layers
     c = kernel_costs(wl, B)
     flops = L * sum(c[k][0] for k in ("qkv", "out_proj", "gate_up", "down", "attention"))
-    flops += c["film"][0] + 2 * c["time_mlp"][0] + c["embed_norm"][0] + c["velocity"][0]
+    flops += c["embed_norm"][0] + c["velocity"][0]
+    if film:
+        flops += c["film"][0] + 2 * c["time_mlp"][0]
     W, F, Dq, dh, A = wl.width, wl.mlp_dim, wl.n_q_heads * wl.head_dim, wl.head_dim, wl.action_dim
-    wbytes = 2.0 * L * ((Dq + 2 * dh) * W + W * Dq + 2 * F * W + W * F)
-    wbytes += 2.0 * (L * 6 * W + 2 * W) * W + 2.0 * 2 * W * W + 4.0 * 2 * A * W
+    wbytes = 2.0 * L * ((Dq + 2 * dh) * W + W * Dq + 2 * F * W + W * F) + 4.0 * 2 * A * W
+    if film:
+        wbytes += 2.0 * (L * 6 * W + 2 * W) * W + 2.0 * 2 * W * W
     kv = 2.0 * L * sum(wl.prefix_lens[:B]) * dh * 2
     return flops, wbytes + kv
 
@@ -216,6 +220,107 @@ def time_oracle(wl, w, pre, buf, tau, budget_s: float, max_steps: int):
     return n, dt, cores
 
 
+_ORACLE_ONE_THREAD = r"""
+import json, os, sys, time
+sys.path.insert(0, sys.argv[1])
+import numpy as np
+import oracle
+import workloads as WL
+wl = WL.standard_workloads()[sys.argv[2]]
+budget = float(sys.argv[3])
+w = WL.make_weights(wl); pre = WL.make_prefix_kv(wl)
+buf, tau = WL.make_buffer(wl), WL.make_noise_levels(wl)
+fresh = np.zeros((wl.batch, wl.chunk_tokens, wl.action_dim), np.float32)
+t0 = time.perf_counter(); oracle.stream_step(w, wl.as_config(), buf, tau, pre, fresh)
+first = time.perf_counter() - t0
+n = int(max(1, min(50, budget // max(first, 1e-9))))
+t0 = time.perf_counter()
+for _ in range(n):
+    oracle.stream_step(w, wl.as_config(), buf, tau, pre, fresh)
+print(json.dumps({"n": n, "dt": time.perf_counter() - t0}))
+"""
+
+
+def time_oracle_one_thread(wl_name: str, budget_s: float):
+    """The oracle on one host core: a child process with every BLAS / OpenMP thread
+    pool limited to one thread (set before NumPy loads)."""
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               BLIS_NUM_THREADS="1", NUMEXPR_NUM_THREADS="1", CUDA_VISIBLE_DEVICES="")
+    try:
+        out = subprocess.run([sys.executable, "-c", _ORACLE_ONE_THREAD, ROOT, wl_name,
+                              str(budget_s)], env=env, capture_output=True, text=True,
+                             timeout=20 * budget_s + 120)
+        r = json.loads(out.stdout.strip().splitlines()[-1])
+        return r["n"], r["dt"]
+    except (OSError, ValueError, IndexError, KeyError, subprocess.TimeoutExpired):
+        return None
+
+
+# ---------------------------------------------------------------------------
+# isolated chunk-causal attention over the prefix sweep (T = 500 action tokens)
+# ---------------------------------------------------------------------------
+
+def attention_sweep(dev, stream, peaks, prefixes=(256, 512, 1024, 2048, 4096), iters=40):
+    """fva_chunk_attention on one layer's inputs (K=10 x H=50 tokens, 8 query heads of
+    256, one KV head) for each prefix length P.  Every launch reads a different copy
+    of K and V, and the copies together exceed the 129 MB L2, so the prefix keys come
+    from HBM as in the step; q (written just before attention in the step) is one
+    copy.  CUDA events on the launching stream."""
+    import torch
+    import paper_2608_27384_gb300 as fva
+    from paper_2608_27384_gb300.harness import config_for
+    K, H, nq, dh = 10, 50, 8, 256
+    T = K * H
+    wl = WL.small_bf16_workload(n_layers=1, n_q_heads=nq, n_chunks=K, chunk_tokens=H,
+                                prefix_lens=[max(prefixes)])
+    h = fva.fva_create(config_for(wl))
+    out_rows = []
+    try:
+        gen = torch.Generator(device=dev).manual_seed(0)
+        q = torch.randn((T * nq, dh), device=dev, generator=gen).to(torch.bfloat16)
+        o = torch.empty_like(q)
+        for P in prefixes:
+            kv_rows = P + T
+            per_copy = 2 * kv_rows * dh * 2
+            n_copy = max(2, -(-160 * 2 ** 20 // per_copy))
+            kp = torch.randn((n_copy, kv_rows, dh), device=dev, generator=gen).to(torch.bfloat16)
+            vp = torch.randn((n_copy, kv_rows, dh), device=dev, generator=gen).to(torch.bfloat16)
+            pl = torch.tensor([P], dtype=torch.int32, device=dev)
+            with torch.cuda.stream(stream):
+                for i in range(3):
+                    fva.fva_chunk_attention(h, q, kp[i % n_copy], vp[i % n_copy], pl, 1, kv_rows,
+                                            o, stream)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                for i in range(iters):
+                    fva.fva_chunk_attention(h, q, kp[i % n_copy], vp[i % n_copy], pl, 1, kv_rows,
+                                            o, stream)
+                e1.record(stream)
+            torch.cuda.synchronize()
+            us = 1e3 * e0.elapsed_time(e1) / iters
+            pairs = P * T + H * H * K * (K + 1) // 2
+            flops = 4.0 * dh * nq * pairs
+            tf = flops / (us * 1e-6) / 1e12
+            out_rows.append({"prefix": P, "us": round(us, 3), "tflops": round(tf, 1),
+                             "frac_of_burst": round(tf / peaks["bf16_tflops"], 4),
+                             "kv_copies": n_copy})
+            del kp, vp
+    finally:
+        fva.fva_destroy(h)
+    return out_rows
+
+
+def ncu_launch_shares(workload):
+    """Per-kind shares of the committed ncu launch list of this workload, if any."""
+    path = os.path.join(ROOT, "profiles", f"step_{workload}_launches.json")
+    try:
+        with open(path) as f:
+            return json.load(f)
+    except (OSError, ValueError):
+        return None
+
+
 # ---------------------------------------------------------------------------
 
 class Replicas:
@@ -272,6 +377,10 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-isolated", action="store_true",
                     help="skip the isolated-decode comparison (K passes over one chunk)")
+    ap.add_argument("--no-sweep", action="store_true",
+                    help="skip the isolated attention prefix sweep")
+    ap.add_argument("--clock-soak", type=float, default=1.5,
+                    help="seconds of untimed steps before the timed region while clocks are sampled")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -292,18 +401,36 @@ def main():
     if args.impl == "reference":
         if rank != 0:
             return 0
+        import oracle
         w = WL.make_weights(wl)
         pre = WL.make_prefix_kv(wl)
         buf, tau = WL.make_buffer(wl), WL.make_noise_levels(wl)
-        n, dt, cores = time_oracle(wl, w, pre, buf, tau, budget_s=60.0, max_steps=args.steps)
+        fresh = np.zeros((wl.batch, wl.chunk_tokens, wl.action_dim), np.float32)
+        step = lambda: oracle.stream_step(w, wl.as_config(), buf, tau, pre, fresh)  # noqa: E731
+        # --warmup untimed steps, then --steps timed ones; if that would take more than
+        # about four minutes, as many of each as fit (the line reports the counts used)
+        t0 = time.perf_counter()
+        step()
+        first = time.perf_counter() - t0
+        fit = max(2, int(240.0 // max(first, 1e-9)))
+        n_warm = max(1, min(args.warmup, fit // 4))
+        n = max(1, min(args.steps, fit - n_warm))
+        for _ in range(n_warm - 1):
+            step()
+        t0 = time.perf_counter()
+        for _ in range(n):
+            step()
+        dt = time.perf_counter() - t0
+        cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
         v = n / dt
         line = {"metric": METRIC, "value": v, "unit": "steps/s", "impl": "reference",
-                "n_gpus": args.gpus, "steps": n, "warmup": 1, "ms_per_step": 1e3 * dt / n,
+                "n_gpus": args.gpus, "steps": n, "warmup": n_warm, "ms_per_step": 1e3 * dt / n,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "f64", "data": "synthetic", "config": cfg_json,
                 "cpu_baseline": {"value": v, "unit": "steps/s", "cores": cores, "kind": "oracle",
-                                 "sample": f"{n} full oracle steps (of {args.steps} requested; "
-                                           "bounded to ~60 s of CPU work)"},
+                                 "sample": f"{n} timed full oracle steps after {n_warm} untimed "
+                                           f"(requested {args.steps} and {args.warmup}; bounded "
+                                           "to ~4 min of CPU work)"},
                 "e2e": {"value": v, "unit": "steps/s", "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}}
         print(json.dumps(line))
@@ -335,8 +462,21 @@ def main():
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
             fva.fva_step(h, d_buf, tau, d_out, B, stream)
-    barrier()
+    torch.cuda.synchronize(dev)
+    # The clocks are sampled every 200 ms from here to the end of the timed region.  A
+    # timed region of a few steps lasts milliseconds, so untimed steps (the clock
+    # soak, not counted anywhere) keep the GPU under the same load for about 1.5 s
+    # before it and the samples describe the clocks the timed steps ran at.
     sampler = ClockSampler(gpu_index_for(local_rank))
+    soak_steps = 0
+    soak_t0 = time.perf_counter()
+    with torch.cuda.stream(stream):
+        while time.perf_counter() - soak_t0 < args.clock_soak:
+            for _ in range(100):
+                fva.fva_step(h, d_buf, tau, d_out, B, stream)
+            soak_steps += 100
+            stream.synchronize()
+    barrier()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
     for _ in range(args.steps):
@@ -371,6 +511,29 @@ def main():
     h2d = buf.nbytes + tau.nbytes
     d2h = h_out.numel() * 4
 
+    # ---- the same step reusing the previous step's FiLM modulation (steady streaming
+    # keeps the noise levels fixed, §3.2): a separately labelled extra number
+    film_cached = None
+    if rank == 0:
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                fva.fva_step_ex(h, d_buf, tau, d_out, B, reuse_film=True, stream=stream)
+            ec0 = torch.cuda.Event(enable_timing=True)
+            ec1 = torch.cuda.Event(enable_timing=True)
+            ec0.record(stream)
+            for _ in range(args.steps):
+                fva.fva_step_ex(h, d_buf, tau, d_out, B, reuse_film=True, stream=stream)
+            ec1.record(stream)
+        torch.cuda.synchronize()
+        us_c = 1e3 * ec0.elapsed_time(ec1) / args.steps
+        fl_c, by_c = step_costs(wl, B, film=False)
+        roof_c = max(fl_c / (peaks["bf16_tflops"] * 1e12), by_c / (peaks["hbm_gbs"] * 1e9))
+        film_cached = {"us_per_step": us_c, "steps_per_s": 1e6 / us_c,
+                       "roofline_us": 1e6 * roof_c, "frac": 1e6 * roof_c / us_c,
+                       "note": "FVA_STEP_REUSE_FILM: the time MLP and FiLM projections of the "
+                               "previous step are reused (noise levels unchanged); not the "
+                               "headline, which recomputes them every step"}
+
     # ---- kernel-by-kernel profile (CUDA events between launches on `stream`)
     per_kind = {}
     launches_per_step = 0
@@ -402,6 +565,8 @@ def main():
         roof = {"bound": "hbm", "achieved": by / avg_s / 1e9, "peak": peaks["hbm_gbs"],
                 "unit": "GB/s"}
     roof["frac"] = roof["achieved"] / roof["peak"]
+    if roof["bound"] == "tensor":
+        roof["frac_of_burst"] = roof["achieved"] / peaks["bf16_tflops"]
     roof.update({"traffic": dram_traffic(args.workload, dom), "kernel": dom,
                  "launches_per_step": n // max(1, args.profile_steps),
                  "avg_launch_us": t_us / n, "avg_launch_us_with_event_nodes": per_kind[dom][0] / n,
@@ -467,12 +632,22 @@ def main():
                     "note": "K passes of the same expert over [prefix ; one chunk] per emitted "
                             "chunk (pi0.5-style decode), against one streaming step"}
 
+    sweep = None
+    if rank == 0 and wl.dtype == "bf16" and not args.no_sweep:
+        sweep = attention_sweep(dev, stream, peaks)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         n_cpu, dt_cpu, cores = time_oracle(wl, w, pre, buf, tau, budget_s=args.cpu_budget,
                                            max_steps=1000)
         cpu = {"value": n_cpu / dt_cpu, "unit": "steps/s", "cores": cores, "kind": "oracle",
-               "sample": f"{n_cpu} full oracle steps of the same workload (fp64 NumPy)"}
+               "sample": f"{n_cpu} full oracle steps of the same workload (fp64 NumPy, BLAS "
+                         f"threads on all {cores} host cores)"}
+        one = time_oracle_one_thread(wl.name, args.cpu_budget / 2)
+        if one is not None:
+            cpu["single_thread"] = {"value": one[0] / one[1], "unit": "steps/s", "cores": 1,
+                                    "sample": f"{one[0]} full oracle steps, every BLAS / OpenMP "
+                                              "pool at one thread"}
 
     dec.close()
     if rank == 0:
@@ -492,6 +667,12 @@ def main():
                                 "(profiled step - timed step) / launches is taken off every "
                                 "launch (roofline.event_node_overhead_us)",
                 "isolated_decode": isolated,
+                "attention_sweep": sweep,
+                "film_cached": film_cached,
+                "ncu_launch_shares": ncu_launch_shares(args.workload),
+                "clock_soak": {"steps": soak_steps, "seconds": args.clock_soak,
+                               "note": "untimed steps between the warm-up and the timed "
+                                       "region, under the clock sampler"},
                 "cpu_baseline": cpu}
         print(json.dumps(line))
     replicas.close()

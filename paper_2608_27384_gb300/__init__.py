@@ -51,7 +51,7 @@ class fva_config(ctypes.Structure):
 
 class fva_step_opts(ctypes.Structure):
     _fields_ = [("fresh_noise", ctypes.c_void_p), ("velocity_out", ctypes.c_void_p),
-                ("trace_layer", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("trace_layer", ctypes.c_int32), ("flags", ctypes.c_uint32),
                 ("trace_out", ctypes.c_void_p), ("n_valid", ctypes.c_void_p)]
 
 
@@ -197,16 +197,20 @@ def fva_step(handle: int, buffer, noise_levels, out_chunk, batch: int, stream=No
     _check(lib().fva_step(handle, _ptr(buffer), tp, _ptr(out_chunk), batch, _stream(stream)))
 
 
+FVA_STEP_REUSE_FILM = 1
+
+
 def fva_step_ex(handle: int, buffer, noise_levels, out_chunk, batch: int, fresh_noise=None,
                 velocity_out=None, trace_layer: int = -1, trace_out=None, stream=None,
-                n_valid=None) -> None:
+                n_valid=None, reuse_film: bool = False) -> None:
     """n_valid: per-request real chunks (cold start), a sequence of ints or None."""
     tau, tp = _tau_ptr(noise_levels)
     nv = None
     if n_valid is not None:
         import numpy as _np
         nv = _np.ascontiguousarray(n_valid, dtype=_np.int32)
-    opts = fva_step_opts(_ptr(fresh_noise), _ptr(velocity_out), trace_layer, 0, _ptr(trace_out),
+    opts = fva_step_opts(_ptr(fresh_noise), _ptr(velocity_out), trace_layer,
+                         FVA_STEP_REUSE_FILM if reuse_film else 0, _ptr(trace_out),
                          nv.ctypes.data if nv is not None else None)
     _check(lib().fva_step_ex(handle, _ptr(buffer), tp, _ptr(out_chunk), batch,
                              ctypes.byref(opts), _stream(stream)))

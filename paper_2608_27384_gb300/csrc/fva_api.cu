@@ -107,6 +107,7 @@ struct GraphEntry {
   float* buffer;
   float* out;
   bool fresh;
+  bool reuse_film;
   cudaGraphExec_t exec;
   uint64_t last_use;
 };
@@ -186,6 +187,10 @@ struct fva_handle {
   cudaStream_t cap_stream = nullptr;
   std::vector<GraphEntry> graphs;
   uint64_t use_clock = 0;
+  // the FiLM modulation in `mod` / `cond` was computed for these noise levels
+  bool film_valid = false;
+  int film_batch = 0;
+  std::vector<float> film_tau;
 
   float* tau_dev() const { return params_dev; }
   // padding tokens (K - n_valid) * H per request of the current step
@@ -676,6 +681,7 @@ extern "C" fva_status fva_load_weights(fva_handle* h, const void* const* tensors
   if (h->warena) cudaFree(h->warena);
   h->warena = nullptr;
   h->weights_loaded = false;
+  h->film_valid = false;
   void* arena = nullptr;
   cudaError_t e = cudaMalloc(&arena, img.size());
   if (e != cudaSuccess) {
@@ -824,6 +830,7 @@ namespace {
 struct StepTrace {
   int layer = -1;
   float* out = nullptr;
+  bool reuse_film = false;  // skip the timestep embedding, time MLP and FiLM projection
 };
 
 // Event before every launch (kernel profiling mode of fva_step_profile).  The
@@ -896,11 +903,10 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   };
 
 
-  // ---- per-chunk FiLM condition and modulation (App. A.4)
-  mark(FVA_K_TIMESTEP_EMBED, -1);
-  launch_temb(h->tau_dev(), h->temb_freq, BK, W, h->temb, bf, s);
-  // a projection with at least two tiles per SM and no K-split runs persistent,
-  // so each tile's epilogue overlaps the next tile's MMAs
+  // ---- per-chunk FiLM condition and modulation (App. A.4); reused from the previous
+  // step when the host saw identical noise levels (FVA_STEP_REUSE_FILM)
+  // a projection with at least two tiles per SM and no K-split runs persistent, so
+  // each tile's epilogue overlaps the next tile's MMAs
   auto gemm = [&](int bn, int mode, const CUtensorMap* ma, const CUtensorMap* mb,
                   const GemmEpi& e, int Mr, int N, int Kd, int splits) {
     const long long tiles = (long long)((Mr + 127) / 128) * (N / bn);
@@ -910,41 +916,45 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   };
   GemmEpi ep{};
   ep.err = h->err_dev;
-  if (bf) {
-    // a few rows: one warp per output column (GEMV); more: the tensor-core GEMM
-    // (the GEMV walks its rows 16 at a time)
-    if (BK <= 32) {
-      mark(FVA_K_TIME_MLP, -1);
-      launch_gemv_silu(h->temb, h->w_t1, h->b_t1, h->t1, BK, W, W, s);
-      mark(FVA_K_TIME_MLP, -1);
-      launch_gemv_silu(h->t1, h->w_t2, h->b_t2, h->cond, BK, W, W, s);
+  if (!tr.reuse_film) {
+    mark(FVA_K_TIMESTEP_EMBED, -1);
+    launch_temb(h->tau_dev(), h->temb_freq, BK, W, h->temb, bf, s);
+    if (bf) {
+      // a few rows: one warp per output column (GEMV); more: the tensor-core GEMM
+      // (the GEMV walks its rows 16 at a time)
+      if (BK <= 32) {
+        mark(FVA_K_TIME_MLP, -1);
+        launch_gemv_silu(h->temb, h->w_t1, h->b_t1, h->t1, BK, W, W, s);
+        mark(FVA_K_TIME_MLP, -1);
+        launch_gemv_silu(h->t1, h->w_t2, h->b_t2, h->cond, BK, W, W, s);
+      } else {
+        GemmEpi et{};
+        et.err = h->err_dev;
+        et.out = h->t1;
+        et.bias = h->b_t1;
+        et.ldo = W;
+        mark(FVA_K_TIME_MLP, -1);
+        CUDA_TRY(launch_tc_gemm(kBnTime, GEMM_BIAS_SILU_BF16, &h->m_temb, &h->m_wt1, et, BK, W, W, 1, s));
+        et.out = h->cond;
+        et.bias = h->b_t2;
+        mark(FVA_K_TIME_MLP, -1);
+        CUDA_TRY(launch_tc_gemm(kBnTime, GEMM_BIAS_SILU_BF16, &h->m_t1, &h->m_wt2, et, BK, W, W, 1, s));
+      }
+      ep.out = h->mod;
+      ep.bias = h->b_mod;
+      ep.ldo = h->N_mod;
+      mark(FVA_K_FILM, -1);
+      CUDA_TRY(BK <= 16 ? launch_tc_gemm_stream(&h->m_cond16, &h->m_wmod, ep, BK, h->N_mod, W,
+                                                h->n_sms, s)
+                         : gemm(kBnFilm, GEMM_BIAS_F32, &h->m_cond, &h->m_wmod, ep, BK, h->N_mod, W, 1));
     } else {
-      GemmEpi et{};
-      et.err = h->err_dev;
-      et.out = h->t1;
-      et.bias = h->b_t1;
-      et.ldo = W;
-      mark(FVA_K_TIME_MLP, -1);
-      CUDA_TRY(launch_tc_gemm(kBnTime, GEMM_BIAS_SILU_BF16, &h->m_temb, &h->m_wt1, et, BK, W, W, 1, s));
-      et.out = h->cond;
-      et.bias = h->b_t2;
-      mark(FVA_K_TIME_MLP, -1);
-      CUDA_TRY(launch_tc_gemm(kBnTime, GEMM_BIAS_SILU_BF16, &h->m_t1, &h->m_wt2, et, BK, W, W, 1, s));
+      launch_f32_gemm((float*)h->temb, W, (float*)h->w_t1, h->c32, W, BK, W, W, s);
+      launch_f32_bias_act(h->c32, h->b_t1, (float*)h->t1, BK, W, true, s);
+      launch_f32_gemm((float*)h->t1, W, (float*)h->w_t2, h->c32, W, BK, W, W, s);
+      launch_f32_bias_act(h->c32, h->b_t2, (float*)h->cond, BK, W, true, s);
+      launch_f32_gemm((float*)h->cond, W, (float*)h->w_mod, h->c32, h->N_mod, BK, h->N_mod, W, s);
+      launch_f32_bias_act(h->c32, h->b_mod, h->mod, BK, h->N_mod, false, s);
     }
-    ep.out = h->mod;
-    ep.bias = h->b_mod;
-    ep.ldo = h->N_mod;
-    mark(FVA_K_FILM, -1);
-    CUDA_TRY(BK <= 16 ? launch_tc_gemm_stream(&h->m_cond16, &h->m_wmod, ep, BK, h->N_mod, W,
-                                              h->n_sms, s)
-                       : gemm(kBnFilm, GEMM_BIAS_F32, &h->m_cond, &h->m_wmod, ep, BK, h->N_mod, W, 1));
-  } else {
-    launch_f32_gemm((float*)h->temb, W, (float*)h->w_t1, h->c32, W, BK, W, W, s);
-    launch_f32_bias_act(h->c32, h->b_t1, (float*)h->t1, BK, W, true, s);
-    launch_f32_gemm((float*)h->t1, W, (float*)h->w_t2, h->c32, W, BK, W, W, s);
-    launch_f32_bias_act(h->c32, h->b_t2, (float*)h->cond, BK, W, true, s);
-    launch_f32_gemm((float*)h->cond, W, (float*)h->w_mod, h->c32, h->N_mod, BK, h->N_mod, W, s);
-    launch_f32_bias_act(h->c32, h->b_mod, h->mod, BK, h->N_mod, false, s);
   }
   if (tr.layer >= 0) launch_to_f32(h->cond, bf, tr_at(o_cond), (long long)BK * W, s);
 
@@ -1109,10 +1119,11 @@ fva_status check_async_error(fva_handle* h, cudaStream_t s) {
   return FVA_OK;
 }
 
-fva_status get_graph(fva_handle* h, int B, float* buffer, float* out, bool fresh,
+fva_status get_graph(fva_handle* h, int B, float* buffer, float* out, bool fresh, bool reuse_film,
                      cudaGraphExec_t* exec) {
   for (auto& g : h->graphs)
-    if (g.batch == B && g.buffer == buffer && g.out == out && g.fresh == fresh) {
+    if (g.batch == B && g.buffer == buffer && g.out == out && g.fresh == fresh &&
+        g.reuse_film == reuse_film) {
       g.last_use = ++h->use_clock;
       *exec = g.exec;
       return FVA_OK;
@@ -1127,7 +1138,9 @@ fva_status get_graph(fva_handle* h, int B, float* buffer, float* out, bool fresh
   }
   cudaGraph_t graph;
   CUDA_TRY(cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal));
-  fva_status st = enqueue_step(h, B, buffer, out, fresh, StepTrace{}, h->cap_stream);
+  StepTrace tr;
+  tr.reuse_film = reuse_film;
+  fva_status st = enqueue_step(h, B, buffer, out, fresh, tr, h->cap_stream);
   cudaError_t e = cudaStreamEndCapture(h->cap_stream, &graph);
   if (st != FVA_OK) {
     if (e == cudaSuccess) cudaGraphDestroy(graph);
@@ -1138,7 +1151,7 @@ fva_status get_graph(fva_handle* h, int B, float* buffer, float* out, bool fresh
   e = cudaGraphInstantiate(&ge, graph, 0);
   cudaGraphDestroy(graph);
   CUDA_TRY(e);
-  h->graphs.push_back(GraphEntry{B, buffer, out, fresh, ge, ++h->use_clock});
+  h->graphs.push_back(GraphEntry{B, buffer, out, fresh, reuse_film, ge, ++h->use_clock});
   *exec = ge;
   return FVA_OK;
 }
@@ -1163,6 +1176,8 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     return fail(FVA_ERR_INVALID_ARG, "trace_layer %d >= n_layers", opts->trace_layer);
   if (opts && opts->trace_layer >= 0 && !opts->trace_out)
     return fail(FVA_ERR_INVALID_ARG, "trace_out is NULL");
+  if (opts && (opts->flags & ~FVA_STEP_REUSE_FILM))
+    return fail(FVA_ERR_INVALID_ARG, "unknown step flags 0x%x", opts->flags);
   if (opts && opts->n_valid)
     for (int r = 0; r < batch; ++r)
       if (opts->n_valid[r] < 1 || opts->n_valid[r] > h->K)
@@ -1217,6 +1232,12 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
   h->ring_used[slot] = true;
 
   const bool fresh = opts && opts->fresh_noise;
+  // the previous step's FiLM modulation is reused only for the same batch and
+  // bit-identical noise levels
+  const size_t n_tau = (size_t)batch * h->K;
+  const bool reuse_film = opts && (opts->flags & FVA_STEP_REUSE_FILM) && !prof && h->film_valid &&
+                          h->film_batch == batch && h->film_tau.size() == n_tau &&
+                          std::memcmp(h->film_tau.data(), noise_levels, n_tau * sizeof(float)) == 0;
   if (fresh)
     CUDA_TRY(cudaMemcpyAsync(h->fresh, opts->fresh_noise,
                              sizeof(float) * batch * h->H * h->A, cudaMemcpyDeviceToDevice, s));
@@ -1251,6 +1272,7 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     CUDA_TRY(cudaGraphLaunch(h->prof_exec, s));
   } else if ((opts && opts->trace_layer >= 0) || (h->cfg.flags & FVA_FLAG_NO_GRAPH)) {
     StepTrace tr;
+    tr.reuse_film = reuse_film;
     if (opts && opts->trace_layer >= 0) {
       tr.layer = opts->trace_layer;
       tr.out = opts->trace_out;
@@ -1258,8 +1280,14 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     if ((st = enqueue_step(h, batch, buffer, out_chunk, fresh, tr, s)) != FVA_OK) return st;
   } else {
     cudaGraphExec_t exec;
-    if ((st = get_graph(h, batch, buffer, out_chunk, fresh, &exec)) != FVA_OK) return st;
+    if ((st = get_graph(h, batch, buffer, out_chunk, fresh, reuse_film, &exec)) != FVA_OK)
+      return st;
     CUDA_TRY(cudaGraphLaunch(exec, s));
+  }
+  if (!reuse_film) {
+    h->film_valid = true;
+    h->film_batch = batch;
+    h->film_tau.assign(noise_levels, noise_levels + n_tau);
   }
   if (opts && opts->velocity_out)
     CUDA_TRY(cudaMemcpyAsync(opts->velocity_out, h->vel,

@@ -336,3 +336,25 @@ def test_persistent_gemm_bitwise():
         a, b = results["persistent"][key], results["per_op"][key]
         assert np.isfinite(a).all()
         assert np.array_equal(a.view(np.uint32), b.view(np.uint32)), key
+
+
+def test_reuse_film_matches_recomputed():
+    """FVA_STEP_REUSE_FILM: with bit-identical noise levels the previous step's FiLM
+    modulation is reused and the step's results are bit-identical to recomputing
+    it; with other levels it is recomputed (and matches the oracle)."""
+    wl = WL.small_bf16_workload(n_chunks=3, prefix_lens=[120])
+    case = Case(wl)
+    try:
+        fresh = WL.make_fresh_noise(wl, 1)[0]
+        a = case.run(fresh=fresh)
+        b = case.run(fresh=fresh, reuse_film=True)
+        for key in ("out", "buffer", "vel"):
+            np.testing.assert_array_equal(a[key], b[key])
+        tau2 = (case.tau * np.float32(0.9)).astype(np.float32)  # other levels: recomputed
+        c = case.run(tau=tau2, fresh=fresh, reuse_film=True)
+        check_step(case, c, case.oracle_step(tau=tau2, fresh=fresh), "bf16")
+        d = case.run(tau=tau2, fresh=fresh, reuse_film=True)    # same levels again: reused
+        for key in ("out", "buffer", "vel"):
+            np.testing.assert_array_equal(c[key], d[key])
+    finally:
+        case.close()
