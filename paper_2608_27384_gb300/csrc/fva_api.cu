@@ -917,14 +917,20 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   GemmEpi ep{};
   ep.err = h->err_dev;
   if (!tr.reuse_film) {
-    mark(FVA_K_TIMESTEP_EMBED, -1);
-    launch_temb(h->tau_dev(), h->temb_freq, BK, W, h->temb, bf, s);
+    // a few rows (bf16): the first time-MLP GEMV computes the timestep embeddings
+    // itself; otherwise they are a kernel of their own
+    const bool gemv = bf && BK <= 32;
+    if (!gemv) {
+      mark(FVA_K_TIMESTEP_EMBED, -1);
+      launch_temb(h->tau_dev(), h->temb_freq, BK, W, h->temb, bf, s);
+    }
     if (bf) {
       // a few rows: one warp per output column (GEMV); more: the tensor-core GEMM
       // (the GEMV walks its rows 16 at a time)
-      if (BK <= 32) {
+      if (gemv) {
         mark(FVA_K_TIME_MLP, -1);
-        launch_gemv_silu(h->temb, h->w_t1, h->b_t1, h->t1, BK, W, W, s);
+        launch_gemv_silu(nullptr, h->w_t1, h->b_t1, h->t1, BK, W, W, s, h->tau_dev(),
+                         h->temb_freq);
         mark(FVA_K_TIME_MLP, -1);
         launch_gemv_silu(h->t1, h->w_t2, h->b_t2, h->cond, BK, W, W, s);
       } else {

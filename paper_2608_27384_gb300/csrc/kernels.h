@@ -68,10 +68,13 @@ void launch_velocity_euler(const StepDims& d, const float* yF, const float* w_ou
                            const unsigned long long* step_idx, cudaStream_t s);
 
 // out = silu(in W^T + bias), bf16 [M, K] x [N, K] -> bf16 [M, N]; K a multiple of 8.
+// With tau != nullptr the input rows are instead the timestep embeddings of tau[0..M)
+// (freq as for launch_temb; K = W), computed inside the kernel.
 // gemv_init sets the shared-memory limit for K (once per handle).
 cudaError_t gemv_init(int K);
 void launch_gemv_silu(const void* in, const void* w, const float* bias, void* out, int M, int N,
-                      int K, cudaStream_t s);
+                      int K, cudaStream_t s, const float* tau = nullptr,
+                      const float2* freq = nullptr);
 
 // (cos, sin) of position x frequency for RoPE, fp32 and rounded to fp16 pairs.
 void launch_rope_table(float2* table, uint32_t* table_h, int n_pos, int dh, float theta,

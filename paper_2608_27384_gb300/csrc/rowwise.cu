@@ -19,17 +19,8 @@ namespace fva {
 // tau * c_hi is split exactly with an fma, its integer part is removed exactly,
 // and sincospi of the small remainder gives sin / cos to fp32 accuracy.
 // ----------------------------------------------------------------------------
-template <typename Act>
-__global__ void temb_kernel(const float* __restrict__ tau, const float2* __restrict__ freq,
-                            int W, Act* __restrict__ out) {
-  const int row = blockIdx.y;
-  const int half = W / 2;
-  pdl_trigger();
-  pdl_wait();
-  const float t = tau[row];
-  const int j = blockIdx.x * blockDim.x + threadIdx.x;
-  if (j >= half) return;
-  const float2 c = freq[j];
+// (sin, cos) of tau * (2 / p_j) half turns, with c = (hi, lo) split of 2 / p_j.
+__device__ __forceinline__ float2 temb_sincos(float t, float2 c) {
   const float p = t * c.x;
   const float p_err = fmaf(t, c.x, -p);      // exact remainder of the product
   const float n = rintf(p);                  // |p| < 2^23: exact
@@ -41,8 +32,22 @@ __global__ void temb_kernel(const float* __restrict__ tau, const float2* __restr
     sn = -sn;
     cs = -cs;
   }
-  out[(size_t)row * W + j] = from_float<Act>(sn);
-  out[(size_t)row * W + half + j] = from_float<Act>(cs);
+  return make_float2(sn, cs);
+}
+
+template <typename Act>
+__global__ void temb_kernel(const float* __restrict__ tau, const float2* __restrict__ freq,
+                            int W, Act* __restrict__ out) {
+  const int row = blockIdx.y;
+  const int half = W / 2;
+  pdl_trigger();
+  pdl_wait();
+  const float t = tau[row];
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= half) return;
+  const float2 sc = temb_sincos(t, freq[j]);
+  out[(size_t)row * W + j] = from_float<Act>(sc.x);
+  out[(size_t)row * W + half + j] = from_float<Act>(sc.y);
 }
 
 void launch_temb(const float* tau, const float2* freq, int rows, int W, void* out,
@@ -113,8 +118,10 @@ inline int row_threads(int W) {
 // R token rows per CTA, so each CTA reads w_in_t (W_in transposed, [A, W] fp32)
 // once for all of them; each thread owns 4 columns of every row.
 // ----------------------------------------------------------------------------
+constexpr int kEmbedMaxA = 32;  // action dims held in registers by the fast path
+
 template <typename Act, int R>
-__global__ void embed_norm_kernel(StepDims d, int rows, const float* __restrict__ buffer,
+__global__ void __launch_bounds__(256) embed_norm_kernel(StepDims d, int rows, const float* __restrict__ buffer,
                                   const float* __restrict__ w_in_t,
                                   const float* __restrict__ b_in, const float* __restrict__ mod,
                                   float* __restrict__ h, Act* __restrict__ y) {
@@ -122,6 +129,66 @@ __global__ void embed_norm_kernel(StepDims d, int rows, const float* __restrict_
   __shared__ float red[32];
   const int m0 = blockIdx.x * R;
   const int nr = min(R, rows - m0);
+  if (d.W == 4 * (int)blockDim.x && d.A <= kEmbedMaxA) {
+    // one float4 column group per thread: W_in (static) is in registers before the
+    // wait for the predecessor; after it one round of loads (this CTA's buffer rows
+    // and their FiLM scale / shift), one CTA-wide reduction for all R rows
+    __shared__ float red_r[R][32];
+    const int col = threadIdx.x * 4;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    float4 wreg[kEmbedMaxA];
+#pragma unroll
+    for (int a = 0; a < kEmbedMaxA; ++a)
+      if (a < d.A) wreg[a] = *reinterpret_cast<const float4*>(w_in_t + (size_t)a * d.W + col);
+    const float4 bias = *reinterpret_cast<const float4*>(b_in + col);
+    pdl_trigger();
+    pdl_wait();
+    for (int i = threadIdx.x; i < R * d.A; i += blockDim.x) {
+      const int r = i / d.A, a = i % d.A;
+      xs[r][a] = r < nr ? buffer[(size_t)(m0 + r) * d.A + a] : 0.f;
+    }
+    float4 sc[R], sh[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      const int m = min(m0 + r, rows - 1);
+      const int rq = m / d.T, c = (m % d.T) / d.H;
+      const float* mrow = mod + (size_t)(rq * d.K + c) * d.N_mod;
+      sc[r] = *reinterpret_cast<const float4*>(mrow + mod_off(0, 0, d.W) + col);
+      sh[r] = *reinterpret_cast<const float4*>(mrow + mod_off(0, 1, d.W) + col);
+    }
+    __syncthreads();
+    float4 acc[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      acc[r] = bias;
+#pragma unroll
+      for (int a = 0; a < kEmbedMaxA; ++a) {
+        if (a >= d.A) break;
+        const float xa = xs[r][a];
+        acc[r].x = fmaf(xa, wreg[a].x, acc[r].x);
+        acc[r].y = fmaf(xa, wreg[a].y, acc[r].y);
+        acc[r].z = fmaf(xa, wreg[a].z, acc[r].z);
+        acc[r].w = fmaf(xa, wreg[a].w, acc[r].w);
+      }
+      if (r < nr) *reinterpret_cast<float4*>(h + (size_t)(m0 + r) * d.W + col) = acc[r];
+      const float ss = warp_sum(acc[r].x * acc[r].x + acc[r].y * acc[r].y +
+                                acc[r].z * acc[r].z + acc[r].w * acc[r].w);
+      if (lane == 0) red_r[r][warp] = ss;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      if (r >= nr) break;
+      float tot = 0.f;
+      for (int w = 0; w < nw; ++w) tot += red_r[r][w];
+      const float rn = rsqrtf(tot / (float)d.W + d.eps);
+      store4<Act>(y + (size_t)(m0 + r) * d.W + col, acc[r].x * rn * (1.f + sc[r].x) + sh[r].x,
+                  acc[r].y * rn * (1.f + sc[r].y) + sh[r].y,
+                  acc[r].z * rn * (1.f + sc[r].z) + sh[r].z,
+                  acc[r].w * rn * (1.f + sc[r].w) + sh[r].w);
+    }
+    return;
+  }
   pdl_trigger();
   pdl_wait();
   // buffer [B, K, H, A] = rows of A, token rows m0 .. m0 + nr - 1 contiguous
@@ -182,8 +249,9 @@ template <typename Act, int R>
 static void launch_embed_norm_r(const StepDims& d, int rows, const float* buffer,
                                 const float* w_in_t, const float* b_in, const float* mod,
                                 float* h, Act* y, cudaStream_t s) {
-  launch_pdl(embed_norm_kernel<Act, R>, dim3((rows + R - 1) / R), dim3(row_threads(d.W)), 0, s,
-             d, rows, buffer, w_in_t, b_in, mod, h, y);
+  // at most 256 threads (the register budget of the fast path); wider rows loop
+  launch_pdl(embed_norm_kernel<Act, R>, dim3((rows + R - 1) / R),
+             dim3(std::min(row_threads(d.W), 256)), 0, s, d, rows, buffer, w_in_t, b_in, mod, h, y);
 }
 
 template <typename Act>
@@ -466,6 +534,13 @@ __global__ void __launch_bounds__(kVelThreads)
   }
   __syncthreads();
   pdl_trigger();
+  // W_out^T does not depend on earlier kernels: with one chunk per CTA its slice is
+  // requested before waiting for the predecessor (the y_F rows after it)
+  const bool one_chunk = wchunk == wq;
+  if (one_chunk && threadIdx.x == 0) {
+    mbar_arrive_expect_tx(&bar, (uint32_t)(sizeof(float) * (d.K + d.A) * wchunk));
+    bulk_load(ws, w_out_t + (size_t)wbeg * d.A, (uint32_t)(sizeof(float) * wchunk * d.A), &bar);
+  }
   pdl_wait();
   const size_t slot = (size_t)d.H * d.A;
   const float* xcol = buffer + ((size_t)r * d.K * d.H + j) * d.A;  // + k*slot selects chunk k
@@ -478,12 +553,14 @@ __global__ void __launch_bounds__(kVelThreads)
     __syncthreads();  // previous chunk consumed
     if (threadIdx.x == 0) {
       // all staging as bulk copies in flight at once: K rows of y_F and the W_out^T slice
-      mbar_arrive_expect_tx(&bar, (uint32_t)(sizeof(float) * (d.K + d.A) * wchunk));
+      if (!one_chunk)
+        mbar_arrive_expect_tx(&bar, (uint32_t)(sizeof(float) * (d.K + d.A) * wchunk));
       for (int k = 0; k < d.K; ++k) {
         const size_t m = (size_t)r * d.T + (size_t)k * d.H + j;
         bulk_load(ys + k * wchunk, yF + m * d.W + w0, sizeof(float) * wchunk, &bar);
       }
-      bulk_load(ws, w_out_t + (size_t)w0 * d.A, (uint32_t)(sizeof(float) * wchunk * d.A), &bar);
+      if (!one_chunk)
+        bulk_load(ws, w_out_t + (size_t)w0 * d.A, (uint32_t)(sizeof(float) * wchunk * d.A), &bar);
     }
     mbar_wait(&bar, phase, nullptr, 0);
     phase ^= 1u;
@@ -541,9 +618,15 @@ __global__ void __launch_bounds__(kVelThreads)
   if (q == 0) {
     const uint32_t vs_addr = smem_u32(vs);
     for (int i = threadIdx.x; i < KA; i += blockDim.x) {
+      // every peer's partial requested before any is added (rank order kept)
+      float pv[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int p = 1; p < 4; ++p)
+        if (p < nsplit) pv[p] = ld_shared_cluster_f32(mapa_shared(vs_addr + 4u * (uint32_t)i, (uint32_t)p));
       float v = vs[i];
-      for (int p = 1; p < nsplit; ++p)
-        v += ld_shared_cluster_f32(mapa_shared(vs_addr + 4u * (uint32_t)i, (uint32_t)p));
+#pragma unroll
+      for (int p = 1; p < 4; ++p)
+        if (p < nsplit) v += pv[p];
       vs[i] = b_out[i % d.A] + v;
     }
   }
@@ -616,49 +699,91 @@ void launch_velocity_euler(const StepDims& d, const float* yF, const float* w_ou
 // each lane reads 8 contiguous weights per 16-byte load.  K a multiple of 8.
 // ----------------------------------------------------------------------------
 constexpr int kGemvRows = 16;
-constexpr int kGemvWarps = 8;
+constexpr int kGemvWarps = 8;    // 4 output columns per CTA, two warps (halves of K) each
+constexpr int kGemvCols = kGemvWarps / 2;
 constexpr int kGemvMaxK8 = 512;  // K <= 4096: each lane keeps its weights in registers
+
+// Sum of v[0..15] over the 32 lanes of the warp for all 16 values at once: four
+// steps that each send half of the lane's values to the partner lane and add the
+// other half (16 values -> 1), then one last exchange.  Lane l ends with the total
+// of value index ((l >> 4) & 1) * 8 + ((l >> 3) & 1) * 4 + ((l >> 2) & 1) * 2 +
+// ((l >> 1) & 1) (both lanes of a pair hold it).  16 shuffles instead of 80.
+__device__ __forceinline__ float warp_sum16(float (&v)[16], int lane) {
+#pragma unroll
+  for (int step = 0; step < 4; ++step) {
+    const int b = 16 >> step, n = 8 >> step;  // partner bit, values kept
+    const bool up = lane & b;
+#pragma unroll
+    for (int i = 0; i < n; ++i) {
+      const float mine = up ? v[i + n] : v[i];
+      const float theirs = up ? v[i] : v[i + n];
+      v[i] = mine + __shfl_xor_sync(0xffffffffu, theirs, b);
+    }
+  }
+  return v[0] + __shfl_xor_sync(0xffffffffu, v[0], 1);
+}
+
+__device__ __forceinline__ int warp_sum16_index(int lane) {
+  return ((lane >> 4) & 1) * 8 + ((lane >> 3) & 1) * 4 + ((lane >> 2) & 1) * 2 + ((lane >> 1) & 1);
+}
 
 __global__ void __launch_bounds__(32 * kGemvWarps)
     gemv_silu_kernel(const bf16* __restrict__ in, const bf16* __restrict__ w,
                      const float* __restrict__ bias, bf16* __restrict__ out, int M, int N,
-                     int K) {
+                     int K, const float* __restrict__ tau, const float2* __restrict__ freq) {
   extern __shared__ __align__(16) uint4 sin4[];  // [16][K/8]
   __shared__ __align__(8) uint64_t bar;
+  __shared__ float part[kGemvCols][kGemvRows];   // the upper K halves' sums
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n = blockIdx.x * kGemvWarps + warp;
-  const int k8 = K / 8;
+  const int col = warp >> 1, khalf = warp & 1;
+  const int n = blockIdx.x * kGemvCols + col;
+  const int k8 = K / 8, k8h = k8 / 2;
   if (threadIdx.x == 0) {
     mbar_init(&bar, 1);
     fence_barrier_init();
   }
   __syncthreads();
-  // this warp's weight row: lane holds chunks lane, lane+32, ... (weights do not
-  // depend on earlier kernels, so they are requested before waiting)
-  uint4 wv[kGemvMaxK8 / 32];
-  const uint4* wr = reinterpret_cast<const uint4*>(w + (size_t)min(n, N - 1) * K);
+  // this warp's half of the weight row: lane holds chunks kh*k8h + lane + 32 i
+  // (the weights do not depend on earlier kernels: requested before waiting)
+  uint4 wv[kGemvMaxK8 / 64];
+  const uint4* wr = reinterpret_cast<const uint4*>(w + (size_t)min(n, N - 1) * K) + khalf * k8h;
 #pragma unroll
-  for (int i = 0; i < kGemvMaxK8 / 32; ++i)
-    if (lane + 32 * i < k8) wv[i] = __ldg(wr + lane + 32 * i);
+  for (int i = 0; i < kGemvMaxK8 / 64; ++i)
+    if (lane + 32 * i < k8h) wv[i] = __ldg(wr + lane + 32 * i);
   pdl_trigger();
   pdl_wait();
+  const float bn = n < N ? bias[n] : 0.f;
   uint32_t phase = 0;
   for (int m0 = 0; m0 < M; m0 += kGemvRows) {
     const int mr = min(kGemvRows, M - m0);
     __syncthreads();
-    if (threadIdx.x == 0) {
-      mbar_arrive_expect_tx(&bar, (uint32_t)(mr * K * 2));
-      bulk_load(sin4, in + (size_t)m0 * K, (uint32_t)(mr * K * 2), &bar);
+    if (tau) {
+      // the input rows are the timestep embeddings of tau[m0 ..]: computed here (the
+      // same arithmetic as temb_kernel) instead of read back from global memory
+      bf16* sinb = reinterpret_cast<bf16*>(sin4);
+      const int half = K / 2;
+      for (int i = threadIdx.x; i < mr * half; i += blockDim.x) {
+        const int mm = i / half, j = i - mm * half;
+        const float2 sc = temb_sincos(tau[m0 + mm], freq[j]);
+        sinb[mm * K + j] = __float2bfloat16_rn(sc.x);
+        sinb[mm * K + half + j] = __float2bfloat16_rn(sc.y);
+      }
+      __syncthreads();
+    } else {
+      if (threadIdx.x == 0) {
+        mbar_arrive_expect_tx(&bar, (uint32_t)(mr * K * 2));
+        bulk_load(sin4, in + (size_t)m0 * K, (uint32_t)(mr * K * 2), &bar);
+      }
+      mbar_wait(&bar, phase, nullptr, 0);
+      phase ^= 1u;
     }
-    mbar_wait(&bar, phase, nullptr, 0);
-    phase ^= 1u;
     float acc[kGemvRows];
 #pragma unroll
     for (int mm = 0; mm < kGemvRows; ++mm) acc[mm] = 0.f;
 #pragma unroll
-    for (int i = 0; i < kGemvMaxK8 / 32; ++i) {
+    for (int i = 0; i < kGemvMaxK8 / 64; ++i) {
       const int c = lane + 32 * i;
-      if (c >= k8) break;
+      if (c >= k8h) break;
       const __nv_bfloat162* w2 = reinterpret_cast<const __nv_bfloat162*>(&wv[i]);
       float wf[8];
 #pragma unroll
@@ -670,21 +795,27 @@ __global__ void __launch_bounds__(32 * kGemvWarps)
 #pragma unroll
       for (int mm = 0; mm < kGemvRows; ++mm) {
         if (mm >= mr) break;
-        const uint4 xv = sin4[mm * k8 + c];
+        const uint4 xv = sin4[mm * k8 + khalf * k8h + c];
         const __nv_bfloat162* x2 = reinterpret_cast<const __nv_bfloat162*>(&xv);
+        float a0 = acc[mm], a1 = 0.f;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const float2 f = __bfloat1622float2(x2[u]);
-          acc[mm] = fmaf(f.x, wf[2 * u], fmaf(f.y, wf[2 * u + 1], acc[mm]));
+        for (int u = 0; u < 4; u += 2) {
+          const float2 f0 = __bfloat1622float2(x2[u]);
+          const float2 f1 = __bfloat1622float2(x2[u + 1]);
+          a0 = fmaf(f0.x, wf[2 * u], a0);
+          a1 = fmaf(f0.y, wf[2 * u + 1], a1);
+          a0 = fmaf(f1.x, wf[2 * u + 2], a0);
+          a1 = fmaf(f1.y, wf[2 * u + 3], a1);
         }
+        acc[mm] = a0 + a1;
       }
     }
-#pragma unroll
-    for (int mm = 0; mm < kGemvRows; ++mm) {
-      const float v = warp_sum(acc[mm]);
-      if (lane == mm && mm < mr && n < N)
-        out[(size_t)(m0 + mm) * N + n] = __float2bfloat16_rn(silu_f(v + bias[n]));
-    }
+    const float tot = warp_sum16(acc, lane);
+    const int mm = warp_sum16_index(lane);
+    if (khalf == 1 && (lane & 1) == 0) part[col][mm] = tot;
+    __syncthreads();
+    if (khalf == 0 && (lane & 1) == 0 && mm < mr && n < N)
+      out[(size_t)(m0 + mm) * N + n] = __float2bfloat16_rn(silu_f(tot + part[col][mm] + bn));
   }
 }
 
@@ -694,11 +825,11 @@ cudaError_t gemv_init(int K) {
 }
 
 void launch_gemv_silu(const void* in, const void* w, const float* bias, void* out, int M, int N,
-                      int K, cudaStream_t s) {
+                      int K, cudaStream_t s, const float* tau, const float2* freq) {
   if (M <= 0) return;
-  launch_pdl(gemv_silu_kernel, dim3((N + kGemvWarps - 1) / kGemvWarps), dim3(32 * kGemvWarps),
+  launch_pdl(gemv_silu_kernel, dim3((N + kGemvCols - 1) / kGemvCols), dim3(32 * kGemvWarps),
              (size_t)kGemvRows * K * 2, s, (const bf16*)in, (const bf16*)w, bias, (bf16*)out, M, N,
-             K);
+             K, tau, freq);
 }
 
 // The bf16 GeGLU epilogue's GELU on an fp32 array (introspection of its accuracy).
