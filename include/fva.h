@@ -72,6 +72,13 @@ typedef enum fva_dtype {
  * is otherwise used where a projection has at least two output tiles per SM (large
  * batches).  Both forms give bit-identical results. */
 #define FVA_FLAG_NO_PERSISTENT_GEMM 4u
+/* bf16: split the attention's keys into fixed-size pieces whose results a second
+ * kernel combines through global scratch, never into a thread-block cluster per query
+ * tile that combines them in distributed shared memory (the form otherwise used when
+ * every query tile's cluster fits on the GPU at once).  Each split's result is rounded
+ * to bf16 before the combination, so the two forms agree to that rounding, and bit for
+ * bit when they cut the keys at the same places. */
+#define FVA_FLAG_NO_ATTN_CLUSTER 8u
 
 /*
  * Shape and numerics of the action expert and of the streaming buffer.

@@ -133,7 +133,7 @@ extern "C" fva_status fva_chunk_attention_noalloc(const void* q, const void* k, 
   a.kv_row0 = 0;
   a.scale_log2 = 1.4426950408889634f / 16.0f;  // log2(e) / sqrt(256)
   a.err = nullptr;
-  cudaError_t e = launch_tc_attention(&mq, &mk, &mv, a, batch, (cudaStream_t)stream);
+  cudaError_t e = launch_tc_attention(&mq, &mk, &mv, a, batch, (cudaStream_t)stream, false);
   if (e == cudaSuccess) e = launch_attn_merge(a, batch, (cudaStream_t)stream);
   if (e != cudaSuccess) return set_error(FVA_ERR_CUDA, cudaGetErrorString(e));
   return FVA_OK;

@@ -128,6 +128,12 @@ struct fva_handle {
   size_t act = 2;  // bytes per activation / weight element
   int W, nq, dh, Dq, F, A, K, H, T, L, Bmax, Pmax, S_cap, N_qkv, N_mod, BKmax, Mmax;
   int tiles_per_req = 0, attn_max_splits = 0, attn_bps = 4;
+  // CTAs per cluster of the attention's cluster form (0: the global form, whose key
+  // splits the merge kernel combines; always so with FVA_FLAG_NO_ATTN_CLUSTER)
+  int attn_ncl = 0;
+  // attn_cluster_capacity by split count (-1: not asked yet)
+  int cluster_cap[kAttnMaxClusterSplits + 1] = {-1, -1, -1, -1, -1, -1, -1, -1, -1};
+  static_assert(kAttnMaxClusterSplits == 8, "initialiser of cluster_cap");
   int n_sms = 0;
   int bn_qkv = kBnQKV, bn_gu = kBnGU;  // tile widths of the QKV and gate/up weight layouts
   // persistent GEMMs where a projection has at least two tiles per SM
@@ -203,6 +209,25 @@ struct fva_handle {
 
 namespace {
 
+// Cluster size of the attention's cluster form for `tiles` query tiles of at most
+// `nkb` 64-key blocks each, or 0 for the global form (splits of `global_bps` blocks
+// and the merge kernel): the largest n <= 8 (and <= nkb) whose clusters the device
+// holds all at once and that leaves every CTA fewer blocks than the global form's
+// splits.  Clusters in a second wave would wait for whole groups of SMs, and every
+// CTA of a cluster stays resident until its tile is combined; the combination
+// through distributed shared memory costs about as much as the merge kernel, so
+// the cluster form pays only with shorter CTAs.
+int attn_cluster_size(fva_handle* h, long long tiles, int nkb, int global_bps) {
+  if (h->cfg.flags & FVA_FLAG_NO_ATTN_CLUSTER) return 0;
+  for (int n = std::min(kAttnMaxClusterSplits, nkb); n >= 2; --n) {
+    const int blocks = (nkb + n - 1) / n;  // fewer CTAs: more blocks each
+    if (blocks > kAttnMaxBlocksPerCta || blocks >= global_bps) break;
+    if (h->cluster_cap[n] < 0) h->cluster_cap[n] = attn_cluster_capacity(n);
+    if (h->cluster_cap[n] >= tiles) return n;
+  }
+  return 0;
+}
+
 fva_status dev_alloc(fva_handle* h, void** p, size_t bytes) {
   if (bytes == 0) bytes = 256;
   cudaError_t e = cudaMalloc(p, bytes);
@@ -265,7 +290,8 @@ fva_status validate_config(const fva_config* c) {
       !std::isfinite(c->rope_theta))
     return fail(FVA_ERR_INVALID_ARG, "bad rms_eps / rope_theta / timestep periods");
   if (c->action_dim > 128) return fail(FVA_ERR_UNSUPPORTED, "action_dim > 128");
-  if (c->flags & ~(FVA_FLAG_NO_GRAPH | FVA_FLAG_BLOCK_DIAGONAL | FVA_FLAG_NO_PERSISTENT_GEMM))
+  if (c->flags & ~(FVA_FLAG_NO_GRAPH | FVA_FLAG_BLOCK_DIAGONAL | FVA_FLAG_NO_PERSISTENT_GEMM |
+                   FVA_FLAG_NO_ATTN_CLUSTER))
     return fail(FVA_ERR_INVALID_ARG, "unknown flags 0x%x", c->flags);
   const long long T = (long long)c->n_chunks * c->chunk_tokens;
   if (T * c->max_batch > (1LL << 24) || c->max_prefix > (1 << 20) || c->n_layers > 1024)
@@ -421,6 +447,7 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
       h->attn_bps /= 2;
     while ((nkb_max + h->attn_bps - 1) / h->attn_bps > 32 && h->attn_bps < 4) h->attn_bps *= 2;
     h->attn_max_splits = (nkb_max + h->attn_bps - 1) / h->attn_bps;
+    h->attn_ncl = attn_cluster_size(h, (long long)h->Bmax * h->tiles_per_req, nkb_max, h->attn_bps);
     const size_t tiles = (size_t)h->Bmax * h->tiles_per_req;
     if ((st = dalloc(h, &h->att_part_o, tiles * h->attn_max_splits * 128 * 256)) ||
         (st = dalloc(h, &h->att_part_ml, tiles * h->attn_max_splits * 128)))
@@ -1020,7 +1047,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       aa.nq = h->nq;
       aa.S_cap = h->S_cap;
       aa.tiles_per_req = h->tiles_per_req;
-      aa.max_splits = h->attn_max_splits;
+      aa.max_splits = h->attn_ncl > 0 ? h->attn_ncl : h->attn_max_splits;
       aa.blocks_per_split = h->attn_bps;
       aa.kv_row0 = l * h->Bmax * h->S_cap;
       aa.scale_log2 = 1.4426950408889634f / std::sqrt((float)h->dh);
@@ -1029,8 +1056,8 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       aa.block_diag = (h->cfg.flags & FVA_FLAG_BLOCK_DIAGONAL) ? 1 : 0;
       aa.prefix_src = h->prefix_src_dev;
       mark(FVA_K_ATTENTION, l);
-      CUDA_TRY(launch_tc_attention(&h->m_q, &h->m_k, &h->m_v, aa, B, s));
-      if (aa.max_splits > 1) {
+      CUDA_TRY(launch_tc_attention(&h->m_q, &h->m_k, &h->m_v, aa, B, s, h->attn_ncl > 0));
+      if (aa.max_splits > 1 && h->attn_ncl == 0) {
         mark(FVA_K_ATTN_MERGE, l);
         CUDA_TRY(launch_attn_merge(aa, B, s));
       }
@@ -1448,7 +1475,11 @@ extern "C" fva_status fva_chunk_attention(fva_handle* h, const void* q, const vo
   aa.kv_row0 = 0;
   aa.scale_log2 = 1.4426950408889634f / std::sqrt((float)h->dh);
   aa.err = h->err_dev;
-  CUDA_TRY(launch_tc_attention(&mq, &mk, &mv, aa, batch, (cudaStream_t)stream));
-  CUDA_TRY(launch_attn_merge(aa, batch, (cudaStream_t)stream));
+  const int ncl = attn_cluster_size(h, (long long)batch * h->tiles_per_req, (kv_rows + 63) / 64,
+                                    aa.blocks_per_split);
+  const bool cluster = ncl > 0;
+  if (cluster) aa.max_splits = ncl;
+  CUDA_TRY(launch_tc_attention(&mq, &mk, &mv, aa, batch, (cudaStream_t)stream, cluster));
+  if (!cluster) CUDA_TRY(launch_attn_merge(aa, batch, (cudaStream_t)stream));
   return FVA_OK;
 }

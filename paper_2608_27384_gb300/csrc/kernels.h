@@ -174,13 +174,24 @@ struct AttnArgs {
 constexpr int kAttnKeysPerSplit = 256;
 constexpr int kAttnKeyBlock = 64;
 
+// Largest cluster of the attention's cluster form (one cluster of CTAs per query
+// tile, the tile's key blocks dealt out evenly, at most kAttnMaxBlocksPerCta each).
+constexpr int kAttnMaxClusterSplits = 8;
+constexpr int kAttnMaxBlocksPerCta = 4;
+
 cudaError_t tc_attention_init();
-// Attention kernel; launch_attn_merge then combines the key splits (it launches
+// How many clusters of `splits` attention CTAs the device can hold at once (0: the
+// cluster form cannot run with that many splits).
+int attn_cluster_capacity(int splits);
+// Attention kernel.  cluster: each query tile is one cluster of a.max_splits CTAs
+// (<= kAttnMaxClusterSplits) that share the tile's key blocks and combine their
+// results inside the cluster; otherwise fixed splits of a.blocks_per_split blocks, and
+// launch_attn_merge then combines them from a.part_o / a.part_ml (it launches
 // nothing when no tile can have more than one split).
 cudaError_t launch_attn_merge(const AttnArgs& a, int B, cudaStream_t s);
 cudaError_t launch_tc_attention(const CUtensorMap* q, const CUtensorMap* k,
                                 const CUtensorMap* v, const AttnArgs& a, int B,
-                                cudaStream_t s);
+                                cudaStream_t s, bool cluster);
 
 // ---------------------------------------------------------------- simt_f32.cu
 // C[M, N] = A[M, K] (lda) * B[N, K]^T, fp32 on CUDA cores.

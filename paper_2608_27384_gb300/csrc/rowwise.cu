@@ -688,7 +688,7 @@ void launch_velocity_euler(const StepDims& d, const float* yF, const float* w_ou
                            const unsigned long long* step_idx, cudaStream_t s) {
   const int ns = vel_split(d);
   launch_pdl_cluster(velocity_euler_kernel, dim3(ns, d.H, d.B), dim3(kVelThreads),
-                     vel_smem_bytes(d), s, ns, d, yF, w_out_t, b_out, dt, buffer, out_chunk,
+                     vel_smem_bytes(d), s, dim3(ns, 1, 1), d, yF, w_out_t, b_out, dt, buffer, out_chunk,
                      vel_out, fresh, seed, step_idx, vel_chunk(d), ns);
 }
 

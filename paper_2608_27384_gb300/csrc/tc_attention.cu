@@ -1,7 +1,4 @@
-// Chunk-wise causal multi-query attention on tcgen05 (head_dim 256, bf16), split-KV
-// form with global scratch.  The step uses attn_cluster_kernel (attention_cluster.cu),
-// which combines its key splits inside a thread-block cluster; this form serves
-// fva_chunk_attention_noalloc, whose scratch is a fixed device array.
+// Chunk-wise causal multi-query attention on tcgen05 (head_dim 256, bf16), split-KV.
 //
 // The paper's mask (§3.1): action token t of chunk c(t) = floor(t / H) attends to
 // every prefix key of its request and to the action keys of chunks <= c(t)
@@ -13,7 +10,7 @@
 // tile in shared memory serves every head.  The key range of a tile is cut into
 // splits of up to 256 keys (1-4 blocks of 64: fewer when there are few query
 // tiles, so that more SMs take part); key blocks past the tile's largest limit
-// are never loaded.  One CTA handles one (tile, split):
+// are never loaded.  One CTA handles one (split, tile):
 //   warp 0      TMA: the Q tile (64 KB) and the split's K blocks, then, once
 //               the S MMAs have read K, the V blocks into the same space;
 //   warp 1      TMEM (512 columns: S in 0..255, O in 256..511); one lane issues
@@ -29,9 +26,22 @@
 // K and V live slab-major: head-dim slab j (64 values, 128 bytes) of key k is
 // at j * 32 KB + k * 128 bytes, so the split's keys form one uniformly strided
 // operand for the S MMA and V's head-dim slabs are 32 KB apart for the P V MMA.
-// A tile with one split writes O / l as bf16.  Otherwise each split writes O / l
-// (bf16) and its (max, sum) to scratch and attn_merge_kernel combines the splits
-// of every row in split order (deterministic) and writes bf16.
+//
+// Two ways to combine the splits of a tile (each split holds O_s / l_s in bf16
+// with its row max m_s and sum l_s):
+//   cluster form: the splits of a tile are one thread-block cluster of n CTAs; the
+//     tile's key blocks are dealt out evenly (CTA s takes blocks
+//     [s nkb / n, (s+1) nkb / n)), at most 4 per CTA.
+//     Each CTA leaves its rows in its own shared memory; after a cluster barrier
+//     CTA q combines rows [q 128/n, (q+1) 128/n) of every split, reading them
+//     through distributed shared memory, and writes the bf16 output rows.
+//     Nothing goes through global scratch and no second kernel runs.
+//   global form (tiles with more splits than a cluster holds, and
+//     fva_chunk_attention_noalloc): each split writes its rows and (m, l) to
+//     global scratch and attn_merge_kernel combines them.
+// Both combine in split order with the same arithmetic, so they give identical
+// bits when they cut the keys at the same places.  A tile with one split writes
+// O / l directly.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -42,19 +52,35 @@ namespace {
 constexpr int kDH = 256;
 constexpr int kRows = 128;
 constexpr int kKB = kAttnKeyBlock;                        // 64 keys per block
-constexpr int kBlocksPerSplit = kAttnKeysPerSplit / kKB;  // 4
+constexpr int kBlocksPerSplit = kAttnKeysPerSplit / kKB;  // 4 K/V slots
+static_assert(kBlocksPerSplit == kAttnMaxBlocksPerCta, "key blocks per CTA");
+constexpr int kGroups = 4;  // softmax threads per query row (16 keys of every block each)
 constexpr int kQBytes = kRows * kDH * 2;                  // 64 KB (Q, later P)
 constexpr int kKVBytes = kKB * kDH * 2;                   // 32 KB per K or V block
 constexpr int kSoftmaxThreads = 512;
 constexpr int kThreads = 64 + kSoftmaxThreads;
 constexpr int kSmem = kQBytes + kBlocksPerSplit * kKVBytes + 1024 /*align*/ + 1024 /*bars*/ +
-                      8 * kRows * 4 /*row exchange*/;
+                      8 * kRows * 4 /*row exchange*/ + kRows * 8 /*row (max, sum)*/;
+// Largest cluster of the cluster form (the portable limit).
+constexpr int kMaxClusterSplits = kAttnMaxClusterSplits;
 constexpr uint32_t kTmemCols = 512;
 
 __device__ __forceinline__ void softmax_bar() {
   asm volatile("bar.sync 1, 512;" ::: "memory");
 }
 
+// Row rr's 16-byte piece c of a split's staged output (cluster form) sits at piece
+// c ^ (rr & 7) of its 512-byte row, so that the 32 rows a warp stages at once
+// fall into different shared-memory banks.
+__device__ __forceinline__ uint32_t stage_piece(int rr, int c) {
+  return (uint32_t)rr * (kDH * 2) + (uint32_t)((c ^ (rr & 7)) << 4);
+}
+
+// Grid (tiles, splits, B).  kCluster: clusters of `splits` CTAs along y, one per
+// query tile (the cluster form); otherwise the global form.
+// 576 threads: 18 warps, 5 of them on two of the SM's four register files (16K
+// registers each), so at most 96 registers a thread.
+template <bool kCluster>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_attn_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
@@ -65,19 +91,30 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int P = __ldg(a.prefix_len + r);
   const int limit_max = attn_key_limit(P, t_last, a.H);
   const int nkb_tile = (limit_max + kKB - 1) / kKB;
+  // splits of this tile: fixed-size ones (global form), or as many CTAs of the
+  // cluster as the tile has key blocks, sharing them evenly (cluster form)
   const int bps = a.blocks_per_split > 0 ? min(a.blocks_per_split, kBlocksPerSplit) : kBlocksPerSplit;
-  const int nsplit = (nkb_tile + bps - 1) / bps;
+  const int nsplit = kCluster ? min((int)gridDim.y, nkb_tile) : (nkb_tile + bps - 1) / bps;
   // a prefix length the KV rows cannot hold (its keys would run into the next
-  // request's rows) or more splits than the scratch holds: the tile is left
-  // unwritten and the error word records it
-  const bool bad = P < 0 || P + a.T > a.S_cap || nsplit > a.max_splits;
-  if (split >= nsplit || bad) {  // uniform over the CTA
-    if (bad && split == 0 && threadIdx.x == 0) report_error(a.err, KERR_BAD_SHAPE);
+  // request's rows), more splits than the scratch holds or more key blocks than
+  // the cluster takes: the tile is left unwritten and the error word records it
+  const bool bad = P < 0 || P + a.T > a.S_cap ||
+                   (kCluster ? nkb_tile > kBlocksPerSplit * (int)gridDim.y
+                             : nsplit > a.max_splits);
+  if (bad) {  // uniform over the tile, hence over its cluster
+    if (split == 0 && threadIdx.x == 0) report_error(a.err, KERR_BAD_SHAPE);
     pdl_trigger();
     return;
   }
-  const int kb0 = split * bps;
-  const int nblk = min(bps, nkb_tile - kb0);
+  // a split past the tile's last key block: nothing to compute (in the cluster
+  // form the CTA still combines its share of the rows)
+  const bool active = split < nsplit;
+  if (!kCluster && !active) {
+    pdl_trigger();
+    return;
+  }
+  const int kb0 = kCluster ? split * nkb_tile / nsplit : split * bps;
+  const int nblk = kCluster ? (split + 1) * nkb_tile / nsplit - kb0 : min(bps, nkb_tile - kb0);
 
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -89,12 +126,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* k_free = bars + 8;    // the S MMAs have read K
   uint64_t* s_full = bars + 9;    // S is in TMEM
   uint64_t* o_full = bars + 10;
-  uint64_t* p_full = bars + 11;   // [4]: P of key block b is in shared memory
+  uint64_t* p_full = bars + 11;   // [4]: P of key block b is in TMEM
   uint32_t* tmem_slot = (uint32_t*)(bars + 15);
-  float* xmax = (float*)(bars + 128);   // [4][128] per-block row max
-  float* xsum = xmax + 4 * kRows;       // [4][128] per-block row sum
+  float* xmax = (float*)(bars + 128);   // [4][128] row max of each key quarter
+  float* xsum = xmax + kGroups * kRows; // [4][128] row sum of each key quarter
+  float2* sml = (float2*)(xsum + kGroups * kRows);  // [128] row (max, sum) of this split (cluster form)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qrow0 = (r * a.T + t0) * a.nq;
+  if (active) {
   if (threadIdx.x == 0) {
     for (int j = 0; j < 4; ++j) mbar_init(&qk_full[j], nblk + 1);  // Q slab + each K block's slab
     for (int b = 0; b < kBlocksPerSplit; ++b) mbar_init(&v_full[b], 1);
@@ -117,7 +157,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tS = tmem, tO = tmem + 256;
   pdl_trigger();
 
-  const int qrow0 = (r * a.T + t0) * a.nq;
   const int krow0 = a.kv_row0 + r * a.S_cap + kb0 * kKB;
   // blocks wholly inside the prefix of a request that shares another's prefix come
   // from that request's rows (same keys; the block that straddles P comes from this
@@ -254,7 +293,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     softmax_bar();
     float mrow = xmax[row];
 #pragma unroll
-    for (int j = 1; j < kBlocksPerSplit; ++j) mrow = fmaxf(mrow, xmax[j * kRows + row]);
+    for (int j = 1; j < kGroups; ++j) mrow = fmaxf(mrow, xmax[j * kRows + row]);
     const float mscaled = mrow > -INFINITY ? mrow * a.scale_log2 : 0.f;
     float l2[2] = {0.f, 0.f};
 #pragma unroll
@@ -295,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     softmax_bar();  // every quarter's sum is in xsum
     l = 0.f;
 #pragma unroll
-    for (int j = 0; j < kBlocksPerSplit; ++j) l += xsum[j * kRows + row];
+    for (int j = 0; j < kGroups; ++j) l += xsum[j * kRows + row];
     const int gtile = r * a.tiles_per_req + tile;
     const int grow = qrow0 + row;  // global q row = (r*T + t) * nq + head
     const int c0 = g * 64;         // O columns of this thread
@@ -320,11 +359,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int u = 0; u < 8; ++u) v[u] = __uint_as_float(ov[8 * i + u]) * inv;
         pk[i] = pack_bf16x8(v);
       }
-      const size_t prow_idx = ((size_t)gtile * a.max_splits + split) * kRows + row;
-      bf16* dst = nsplit == 1 ? (bf16*)a.out + (size_t)grow * kDH + c0
-                              : (bf16*)a.part_o + prow_idx * kDH + c0;
-      warp_store_rows<128>(stage, pk, valid ? dst : nullptr, lane);
-      if (nsplit > 1 && valid && g == 0) __stcg(a.part_ml + prow_idx, make_float2(mx, l));
+      if (kCluster && nsplit > 1) {
+        // cluster form: the rows stay in this CTA's shared memory (Q is dead)
+        // for the combination after the cluster barrier
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+          *reinterpret_cast<uint4*>(sQP + stage_piece(row, g * 8 + i)) = pk[i];
+        if (g == 0) sml[row] = make_float2(mx, l);
+      } else {
+        const size_t prow_idx = ((size_t)gtile * a.max_splits + split) * kRows + row;
+        bf16* dst = nsplit == 1 ? (bf16*)a.out + (size_t)grow * kDH + c0
+                                : (bf16*)a.part_o + prow_idx * kDH + c0;
+        warp_store_rows<128>(stage, pk, valid ? dst : nullptr, lane);
+        if (nsplit > 1 && valid && g == 0) __stcg(a.part_ml + prow_idx, make_float2(mx, l));
+      }
     }
   }
   // the producer and MMA lanes rejoin their warps first: a CTA barrier reached
@@ -335,6 +383,58 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
+  }
+  } else {
+    // inactive split of the cluster form: its output rows come after the QKV
+    // projection's reads of them are over
+    pdl_trigger();
+    pdl_wait();
+  }
+  if constexpr (kCluster) {
+    if (nsplit > 1) {
+      // every split's rows and (max, sum) are staged (release / acquire across the
+      // cluster); CTA `split` then combines rows [split 128/n, (split+1) 128/n)
+      // with attn_merge_kernel's arithmetic, reading the splits through
+      // distributed shared memory, one warp per row and 8 head dims per lane
+      cluster_sync();
+      const int ncl = gridDim.y;  // the cluster: this tile's CTAs, ranks 0..ncl-1 = split
+      const int r_lo = split * kRows / ncl, r_hi = (split + 1) * kRows / ncl;
+      for (int rr = r_lo + warp; rr < r_hi; rr += kThreads / 32) {
+        if (t0 + rr / a.nq >= a.T) break;  // rows past the last token
+        float2 ml = make_float2(-INFINITY, 0.f);
+        if (lane < nsplit) ml = ld_shared_cluster_f2(mapa_shared(smem_u32(&sml[rr]), (uint32_t)lane));
+        const uint32_t piece = smem_u32(sQP + stage_piece(rr, lane));
+        uint4 x[kMaxClusterSplits];
+#pragma unroll
+        for (int u = 0; u < kMaxClusterSplits; ++u)
+          if (u < nsplit) x[u] = ld_shared_cluster_v4(mapa_shared(piece, (uint32_t)u));
+        const float m_all = warp_max(ml.y > 0.f ? ml.x : -INFINITY);
+        // each split holds O_s / l_s; its weight is 2^((m_s - m) c) l_s
+        const float w = ml.y > 0.f ? exp2f((ml.x - m_all) * a.scale_log2) * ml.y : 0.f;
+        const float tot = warp_sum(w);
+        const float inv = tot > 0.f ? 1.f / tot : 0.f;  // no visible key in any split: zeros
+        float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int u = 0; u < kMaxClusterSplits; ++u) {
+          const float wu = __shfl_sync(0xffffffffu, w, u);
+          if (u < nsplit) {
+            const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&x[u]);
+#pragma unroll
+            for (int q2 = 0; q2 < 4; ++q2) {
+              const float2 f = __bfloat1622float2(h2[q2]);
+              acc[2 * q2] = fmaf(wu, f.x, acc[2 * q2]);
+              acc[2 * q2 + 1] = fmaf(wu, f.y, acc[2 * q2 + 1]);
+            }
+          }
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i] *= inv;
+        *reinterpret_cast<uint4*>((bf16*)a.out + (size_t)(qrow0 + rr) * kDH + lane * 8) =
+            pack_bf16x8(acc);
+      }
+      // no CTA leaves (releasing its shared memory) while another still reads it
+      cluster_sync();
+    }
   }
 }
 
@@ -408,15 +508,46 @@ __global__ void __launch_bounds__(256) attn_merge_kernel(const AttnArgs a) {
 }  // namespace
 
 cudaError_t tc_attention_init() {
-  return cudaFuncSetAttribute(tc_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+  cudaError_t e = cudaFuncSetAttribute(tc_attn_kernel<false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(tc_attn_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kSmem);
+  return e;
+}
+
+int attn_cluster_capacity(int splits) {
+  if (splits < 1 || splits > kMaxClusterSplits) return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(1, splits, 1);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = splits;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, tc_attn_kernel<true>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
 }
 
 cudaError_t launch_tc_attention(const CUtensorMap* q, const CUtensorMap* k,
                                 const CUtensorMap* v, const AttnArgs& a, int B,
-                                cudaStream_t s) {
+                                cudaStream_t s, bool cluster) {
+  if (cluster) {
+    if (a.max_splits < 1 || a.max_splits > kMaxClusterSplits) return cudaErrorInvalidValue;
+    return launch_pdl_cluster(tc_attn_kernel<true>, dim3(a.tiles_per_req, a.max_splits, B),
+                              dim3(kThreads), kSmem, s, dim3(1, a.max_splits, 1), *q, *k, *v, a);
+  }
   if (a.max_splits > 32) return cudaErrorInvalidValue;  // the merge holds one split per lane
-  return launch_pdl(tc_attn_kernel, dim3(a.tiles_per_req, a.max_splits, B), dim3(kThreads),
-                    kSmem, s, *q, *k, *v, a);
+  return launch_pdl(tc_attn_kernel<false>, dim3(a.tiles_per_req, a.max_splits, B),
+                    dim3(kThreads), kSmem, s, *q, *k, *v, a);
 }
 
 cudaError_t launch_attn_merge(const AttnArgs& a, int B, cudaStream_t s) {

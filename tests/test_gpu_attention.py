@@ -41,12 +41,12 @@ def oracle_attention(q, k, v, prefix_lens, K, H, nq, dh=256):
     return np.concatenate(out)
 
 
-def make_handle(prefix_lens, K, H, nq, max_prefix=None):
+def make_handle(prefix_lens, K, H, nq, max_prefix=None, flags=0):
     import paper_2608_27384_gb300 as fva
     from paper_2608_27384_gb300.harness import config_for
     wl = WL.small_bf16_workload(n_q_heads=nq, n_chunks=K, chunk_tokens=H, batch=len(prefix_lens),
                                 prefix_lens=list(prefix_lens))
-    return fva.fva_create(config_for(wl, max_prefix=max_prefix))
+    return fva.fva_create(config_for(wl, max_prefix=max_prefix, flags=flags))
 
 
 def run_gpu_attention(handle, q, k, v, prefix_lens, kv_rows):
@@ -98,3 +98,31 @@ def test_chunk_attention_rejects_bad_arguments():
         assert e.value.name == "FVA_ERR_INVALID_ARG"
     finally:
         fva.fva_destroy(h)
+
+
+@pytest.mark.parametrize("prefix_lens,K,H,nq", [
+    ([816], 5, 50, 8),           # 16 query tiles of up to 17 key blocks: clusters of 6, 2-3 blocks each
+    ([37, 300, 611], 3, 50, 8),  # 30 tiles of up to 12 blocks: clusters of 4, the short request's
+                                 # tiles with fewer blocks than CTAs (some CTAs idle)
+    ([129], 3, 50, 4),           # 5 tiles of 32 tokens, 5 blocks: clusters of 5, one block each
+    ([700], 2, 50, 16),          # 13 tiles of 8 tokens, 13 blocks: clusters of 8
+    ([5, 0], 2, 50, 2),          # 4 tiles of 64 tokens, 2 blocks: clusters of 2
+])
+def test_cluster_combination(prefix_lens, K, H, nq):
+    """The key blocks of each query tile shared out over a thread-block cluster and
+    combined in distributed shared memory: matches the oracle, and the global-scratch
+    form with its merge kernel to the bf16 rounding of the split results."""
+    import paper_2608_27384_gb300 as fva
+    q, k, v, kv_rows = attention_inputs(prefix_lens, K, H, nq, seed=3)
+    got = {}
+    for name, flags in (("cluster", 0), ("global", fva.FVA_FLAG_NO_ATTN_CLUSTER)):
+        h = make_handle(prefix_lens, K, H, nq, flags=flags)
+        try:
+            got[name] = run_gpu_attention(h, q, k, v, prefix_lens, kv_rows)
+        finally:
+            fva.fva_destroy(h)
+    ref = oracle_attention(q, k, v, prefix_lens, K, H, nq)
+    assert_close(got["cluster"], ref, max_abs=2e-2, rel_l2=1e-2, what=f"cluster P={prefix_lens}")
+    assert_close(got["global"], ref, max_abs=2e-2, rel_l2=1e-2, what=f"global P={prefix_lens}")
+    assert_close(got["cluster"], got["global"], max_abs=2e-2, rel_l2=5e-3,
+                 what=f"cluster vs global P={prefix_lens}")

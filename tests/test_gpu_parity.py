@@ -306,9 +306,10 @@ def test_step_profile_matches_step_and_counts_launches():
         kinds = [k for k, _, _ in recs]
         L = wl.n_layers
         # 2 time-MLP layers (the first computes the timestep embedding itself), FiLM,
-        # embed+norm; per layer QKV, attention, split merge (prefix 600 + 200 keys >
-        # 256), O-projection, norm, gate/up, down, norm (last layer: final norm);
-        # velocity
+        # embed+norm; per layer QKV, attention, split merge (prefix 600 + 200 keys:
+        # 13 query tiles of 13 key blocks in splits of 2; a cluster of 8 would leave
+        # its CTAs as many blocks, so the global form), O-projection, norm, gate/up,
+        # down, norm (last layer: final norm); velocity
         assert kinds.count("attention") == L and kinds.count("attn_merge") == L, kinds
         assert kinds[-1] == "velocity" and "timestep_embed" not in kinds
         assert len(recs) == 4 + 8 * L + 1, kinds
@@ -337,6 +338,35 @@ def test_persistent_gemm_bitwise():
         a, b = results["persistent"][key], results["per_op"][key]
         assert np.isfinite(a).all()
         assert np.array_equal(a.view(np.uint32), b.view(np.uint32)), key
+
+
+def test_attention_cluster_step():
+    """A step whose attention shares each query tile's key blocks out over a
+    thread-block cluster (16 query tiles of up to 17 key blocks: clusters of 6 CTAs
+    with at most 3 blocks each, against splits of 4 blocks in the global form) and
+    combines them in distributed shared memory, with no merge kernel: matches the
+    oracle, and the step with the global form to the bf16 rounding of the split
+    results."""
+    import torch
+    import paper_2608_27384_gb300 as fva
+    wl = WL.small_bf16_workload(n_chunks=5, prefix_lens=[816])
+    fresh = WL.make_fresh_noise(wl, 1)[0]
+    results = {}
+    for mode, flags in (("cluster", 0), ("merge", fva.FVA_FLAG_NO_ATTN_CLUSTER)):
+        case = Case(wl, flags=flags)
+        try:
+            results[mode] = case.run(fresh=fresh)
+            check_step(case, results[mode], case.oracle_step(fresh=fresh), "bf16")
+            d_buf = case.dev(case.buf)
+            d_out = torch.empty((1, wl.chunk_tokens, wl.action_dim), device="cuda")
+            kinds = [k for k, _, _ in fva.fva_step_profile(case.handle, d_buf, case.tau, d_out, 1)]
+            assert kinds.count("attn_merge") == (0 if mode == "cluster" else wl.n_layers), kinds
+        finally:
+            case.close()
+    for key in ("out", "buffer", "vel"):
+        assert np.isfinite(results["cluster"][key]).all()
+        assert_close(results["cluster"][key], results["merge"][key], rel_l2=5e-3,
+                     what=f"cluster vs merge: {key}")
 
 
 def test_reuse_film_matches_recomputed():
