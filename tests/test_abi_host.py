@@ -25,7 +25,7 @@ def fva():
 def header_functions():
     text = open(os.path.join(ROOT, "include", "fva.h")).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(fva_[a-z_]+)\s*\(", text)))
+    return sorted(set(re.findall(r"\b(fva_[a-z0-9_]+)\s*\(", text)))
 
 
 def test_exports_every_declared_symbol(fva):
