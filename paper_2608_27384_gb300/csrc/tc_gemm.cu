@@ -85,9 +85,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     // B are requested before waiting for the predecessor grid.  A (activations)
     // and everything downstream of it come after the wait; the MMA and epilogue
     // threads only run behind these loads, so they are ordered after it too.
+    // a 64-row A box (every row fits 64) writes half the A stage: the MMA's
+    // rows 64..127 then read stale shared memory and are never stored
+    const uint32_t stage_tx = (uint32_t)(ep.a_rows > 0 ? ep.a_rows : kBM) * kBK * 2 + C::kBBytes;
     const int pre = min(nkb, C::kStages);
     for (int i = 0; i < pre; ++i) {
-      mbar_arrive_expect_tx(&full[i], C::kStageBytes);
+      mbar_arrive_expect_tx(&full[i], stage_tx);
       tma_load_2d(smem + i * C::kStageBytes + C::kABytes, &tmB, (kb0 + i) * kBK, n0, &full[i]);
     }
     pdl_wait();
@@ -98,7 +101,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t ph = (uint32_t)(i / C::kStages) & 1u;
       if (!mbar_wait(&empty[s], ph ^ 1u, ep.err, KERR_WAIT_MMA)) break;
       uint8_t* sa = smem + s * C::kStageBytes;
-      mbar_arrive_expect_tx(&full[s], C::kStageBytes);
+      mbar_arrive_expect_tx(&full[s], stage_tx);
       tma_load_2d(sa, &tmA, (kb0 + i) * kBK, m0, &full[s]);
       tma_load_2d(sa + C::kABytes, &tmB, (kb0 + i) * kBK, n0, &full[s]);
     }
