@@ -79,12 +79,12 @@ typedef enum fva_dtype {
  * to bf16 before the combination, so the two forms agree to that rounding, and bit for
  * bit when they cut the keys at the same places. */
 #define FVA_FLAG_NO_ATTN_CLUSTER 8u
-/* bf16, every row of the step within 64 (max_batch * K * H <= 64, e.g. the paper's
- * 4 x 10 and 5 x 10 buffers): the QKV and gate/up projections load their activation
- * tile through 128-row boxes, most of them zero padding, instead of 64-row boxes
- * (the MMA still runs 128 rows; rows 64..127 are never stored).  Both give
- * bit-identical results. */
-#define FVA_FLAG_NO_Y64 16u
+/* bf16, fewer than 128 rows in the step (max_batch * K * H < 128, e.g. the paper's
+ * 4 x 10, 4 x 20 and 5 x 10 buffers): the QKV and gate/up projections load their
+ * activation tile through 128-row boxes, mostly zero padding, instead of boxes of the
+ * row count rounded up to 16 (the MMA still runs 128 rows; the rows past the box are
+ * never stored).  Both give bit-identical results. */
+#define FVA_FLAG_FULL_A_BOX 16u
 
 /*
  * Shape and numerics of the action expert and of the streaming buffer.

@@ -24,7 +24,7 @@ FVA_FLAG_NO_GRAPH = 1
 FVA_FLAG_BLOCK_DIAGONAL = 2
 FVA_FLAG_NO_PERSISTENT_GEMM = 4
 FVA_FLAG_NO_ATTN_CLUSTER = 8
-FVA_FLAG_NO_Y64 = 16
+FVA_FLAG_FULL_A_BOX = 16
 FVA_PARAM_RING = 8
 
 STATUS = {0: "FVA_OK", 1: "FVA_ERR_INVALID_ARG", 2: "FVA_ERR_STATE", 3: "FVA_ERR_OOM",

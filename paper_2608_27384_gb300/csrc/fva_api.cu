@@ -170,10 +170,11 @@ struct fva_handle {
   int* err_dev = nullptr;
   CUtensorMap m_temb, m_t1, m_cond, m_y, m_attn, m_mlp, m_q, m_k, m_v;
   CUtensorMap m_cond16;  // cond with 16-row boxes (streaming FiLM GEMM)
-  // Every row in 64 (Mmax <= 64, the paper's own buffer shapes): the QKV and gate/up
-  // projections read y through 64-row boxes (FVA_FLAG_NO_Y64: never)
-  bool y64 = false;
-  CUtensorMap m_y64;
+  // Fewer than 128 rows (Mmax < 128, the paper's own buffer shapes): the QKV and
+  // gate/up projections read y through boxes of y_box = Mmax rounded up to 16 rows
+  // (FVA_FLAG_FULL_A_BOX: 128-row boxes); 0 = 128-row boxes
+  int y_box = 0;
+  CUtensorMap m_ybox;
   // per-step parameters: [tau BKmax | dt BKmax | step u64]
   float* params_dev = nullptr;
   float* params_host = nullptr;  // pinned ring [FVA_PARAM_RING][params_floats]
@@ -295,7 +296,7 @@ fva_status validate_config(const fva_config* c) {
     return fail(FVA_ERR_INVALID_ARG, "bad rms_eps / rope_theta / timestep periods");
   if (c->action_dim > 128) return fail(FVA_ERR_UNSUPPORTED, "action_dim > 128");
   if (c->flags & ~(FVA_FLAG_NO_GRAPH | FVA_FLAG_BLOCK_DIAGONAL | FVA_FLAG_NO_PERSISTENT_GEMM |
-                   FVA_FLAG_NO_ATTN_CLUSTER | FVA_FLAG_NO_Y64))
+                   FVA_FLAG_NO_ATTN_CLUSTER | FVA_FLAG_FULL_A_BOX))
     return fail(FVA_ERR_INVALID_ARG, "unknown flags 0x%x", c->flags);
   const long long T = (long long)c->n_chunks * c->chunk_tokens;
   if (T * c->max_batch > (1LL << 24) || c->max_prefix > (1 << 20) || c->n_layers > 1024)
@@ -499,14 +500,17 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
         (st = make_map(&h->m_cond, h->cond, BK, h->W, 128)) ||
         (st = make_map(&h->m_cond16, h->cond, BK, h->W, 16)) ||
         (st = make_map(&h->m_y, h->y, M, h->W, 128)) ||
-        (st = make_map(&h->m_y64, h->y, M, h->W, 64)) ||
+
         (st = make_map(&h->m_attn, h->attn, M, h->Dq, 128)) ||
         (st = make_map(&h->m_mlp, h->mlp, M, h->F, 128)) ||
         (st = make_map(&h->m_q, h->q, M * h->nq, h->dh, 128)) ||
         (st = make_map(&h->m_k, h->kc, (uint64_t)h->L * h->Bmax * h->S_cap, h->dh, 64)) ||
         (st = make_map(&h->m_v, h->vc, (uint64_t)h->L * h->Bmax * h->S_cap, h->dh, 64)))
       return st;
-    h->y64 = M <= 64 && !(h->cfg.flags & FVA_FLAG_NO_Y64);
+    if (M < 128 && !(h->cfg.flags & FVA_FLAG_FULL_A_BOX)) {
+      h->y_box = (int)((M + 15) / 16 * 16);
+      if ((st = make_map(&h->m_ybox, h->y, M, h->W, h->y_box))) return st;
+    }
   }
   CUDA_TRY(cudaDeviceSynchronize());
   return FVA_OK;
@@ -1030,8 +1034,8 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.nq = h->nq;
       ep.dh = h->dh;
       mark(FVA_K_QKV, l);
-      if (h->y64) ep.a_rows = 64;
-      CUDA_TRY(gemm(h->bn_qkv, GEMM_QKV_ROPE, h->y64 ? &h->m_y64 : &h->m_y, &lw.m_qkv, ep, M,
+      ep.a_rows = h->y_box;
+      CUDA_TRY(gemm(h->bn_qkv, GEMM_QKV_ROPE, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_qkv, ep, M,
                     h->N_qkv, W, 1));
     } else {
       launch_f32_gemm((float*)h->y, W, (float*)lw.w_qkv, h->c32, h->N_qkv, M, h->N_qkv, W, s);
@@ -1101,8 +1105,8 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.out = h->mlp;
       ep.ldo = F;
       mark(FVA_K_GATE_UP, l);
-      if (h->y64) ep.a_rows = 64;
-      CUDA_TRY(gemm(h->bn_gu, GEMM_GEGLU, h->y64 ? &h->m_y64 : &h->m_y, &lw.m_gu, ep, M, 2 * F,
+      ep.a_rows = h->y_box;
+      CUDA_TRY(gemm(h->bn_gu, GEMM_GEGLU, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_gu, ep, M, 2 * F,
                     W, 1));
       ep.a_rows = 0;
       ep.out = h->part;

@@ -117,8 +117,9 @@ struct GemmEpi {
   const uint32_t* rope_h;  // the same table as fp16 (cos, sin) pairs
   int T, S_cap, nq, dh;
   int* err;
-  // rows of the A box (the activation tile) the kernel waits for: 0 = 128; 64 when
-  // every row fits 64 (the MMA still reads 128 rows; rows 64..127 are never stored)
+  // rows of the A box (the activation tile) the kernel waits for: 0 = 128; fewer (a
+  // multiple of 16) when every row fits them (the MMA still reads 128 rows; the rows
+  // past the box are never stored)
   int a_rows;
 };
 

@@ -85,8 +85,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // B are requested before waiting for the predecessor grid.  A (activations)
     // and everything downstream of it come after the wait; the MMA and epilogue
     // threads only run behind these loads, so they are ordered after it too.
-    // a 64-row A box (every row fits 64) writes half the A stage: the MMA's
-    // rows 64..127 then read stale shared memory and are never stored
+    // a short A box (every row fits a_rows < 128) writes part of the A stage: the
+    // MMA's later rows then read stale shared memory and are never stored
     const uint32_t stage_tx = (uint32_t)(ep.a_rows > 0 ? ep.a_rows : kBM) * kBK * 2 + C::kBBytes;
     const int pre = min(nkb, C::kStages);
     for (int i = 0; i < pre; ++i) {

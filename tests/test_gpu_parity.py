@@ -370,20 +370,21 @@ def test_attention_cluster_step():
 
 
 @pytest.mark.parametrize("wl_kw", [
-    dict(n_chunks=4, chunk_tokens=10, prefix_lens=[200]),              # 40 rows
+    dict(n_chunks=4, chunk_tokens=10, prefix_lens=[200]),              # 40 rows: 48-row boxes
     dict(batch=2, n_chunks=3, chunk_tokens=8, prefix_lens=[30, 70]),   # 48 rows of two requests
-    dict(n_chunks=2, chunk_tokens=32, prefix_lens=[90]),               # exactly 64 rows
+    dict(n_chunks=4, chunk_tokens=20, prefix_lens=[90]),               # 80 rows: 80-row boxes
+    dict(n_chunks=2, chunk_tokens=63, prefix_lens=[50]),               # 126 rows: 128-row boxes
 ])
-def test_y64_boxes_bitwise(wl_kw):
-    """Every row within 64: the QKV and gate/up projections that load their
-    activation tile through 64-row boxes (the MMA's rows 64..127 then read stale
-    shared memory and are never stored) give the bits of 128-row boxes and match the
-    oracle."""
+def test_short_a_boxes_bitwise(wl_kw):
+    """Fewer than 128 rows: the QKV and gate/up projections that load their
+    activation tile through boxes of the row count rounded up to 16 (the MMA's later
+    rows then read stale shared memory and are never stored) give the bits of
+    128-row boxes and match the oracle."""
     import paper_2608_27384_gb300 as fva
     wl = WL.small_bf16_workload(**wl_kw)
     fresh = WL.make_fresh_noise(wl, 1)[0]
     results = {}
-    for mode, flags in (("y64", 0), ("y128", fva.FVA_FLAG_NO_Y64)):
+    for mode, flags in (("short", 0), ("full", fva.FVA_FLAG_FULL_A_BOX)):
         case = Case(wl, flags=flags)
         try:
             results[mode] = case.run(fresh=fresh)
@@ -391,7 +392,7 @@ def test_y64_boxes_bitwise(wl_kw):
         finally:
             case.close()
     for key in ("out", "buffer", "vel"):
-        a, b = results["y64"][key], results["y128"][key]
+        a, b = results["short"][key], results["full"][key]
         assert np.isfinite(a).all()
         assert np.array_equal(a.view(np.uint32), b.view(np.uint32)), key
 
