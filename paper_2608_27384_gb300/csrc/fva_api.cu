@@ -988,7 +988,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.ldo = h->N_mod;
       mark(FVA_K_FILM, -1);
       CUDA_TRY(BK <= 16 ? launch_tc_gemm_stream(&h->m_cond16, &h->m_wmod, ep, BK, h->N_mod, W,
-                                                h->n_sms, s)
+                                                2 * h->n_sms, s)
                          : gemm(kBnFilm, GEMM_BIAS_F32, &h->m_cond, &h->m_wmod, ep, BK, h->N_mod, W, 1));
     } else {
       launch_f32_gemm((float*)h->temb, W, (float*)h->w_t1, h->c32, W, BK, W, W, s);

@@ -149,8 +149,9 @@ cudaError_t launch_tc_gemm_persist(int bn, int mode, const CUtensorMap* a, const
                                    const GemmEpi& ep, int M, int N, int K, int grid,
                                    cudaStream_t s);
 
-// Persistent weight-streaming form of (kBnFilm, BIAS_F32) for M <= 128 rows: at
-// most `grid` CTAs (one per SM) walk the N / kBnFilm column tiles.
+// Persistent weight-streaming form of (kBnFilm, BIAS_F32) for M <= 16 rows: at
+// most `grid` CTAs (two per SM: pass twice the SM count) walk the N / kBnFilm
+// column tiles.
 cudaError_t launch_tc_gemm_stream(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep,
                                   int M, int N, int K, int grid, cudaStream_t s);
 
