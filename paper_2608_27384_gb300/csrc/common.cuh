@@ -120,6 +120,12 @@ __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
 
+// Ask L2 to fetch `bytes` (a multiple of 16) of global memory from `gsrc`
+// (16-byte aligned); no completion to wait for.
+__device__ __forceinline__ void prefetch_l2(const void* gsrc, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(gsrc), "r"(bytes) : "memory");
+}
+
 // Plain bulk copy global -> shared (both 16-byte aligned, bytes a multiple of
 // 16), completing on `bar` with complete_tx.
 __device__ __forceinline__ void bulk_load(void* smem_dst, const void* gsrc, uint32_t bytes,

@@ -1033,6 +1033,14 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.S_cap = h->S_cap;
       ep.nq = h->nq;
       ep.dh = h->dh;
+      // this layer's FiLM modulation rows (scale, shift, gate of both norms, 6W
+      // floats per chunk), written at the start of the step and long evicted from
+      // L2 by the weights streamed since: L2 fetches them while the QKV projection
+      // runs, ahead of the layer's two residual + norm kernels
+      ep.pf_base = h->mod + mod_off(l, 0, W);
+      ep.pf_count = BK;
+      ep.pf_bytes = 6 * W * (int)sizeof(float);
+      ep.pf_stride = h->N_mod;
       mark(FVA_K_QKV, l);
       ep.a_rows = h->y_box;
       CUDA_TRY(gemm(h->bn_qkv, GEMM_QKV_ROPE, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_qkv, ep, M,

@@ -121,6 +121,11 @@ struct GemmEpi {
   // multiple of 16) when every row fits them (the MMA still reads 128 rows; the rows
   // past the box are never stored)
   int a_rows;
+  // optional L2 prefetch issued by the first CTA before its dependency wait:
+  // pf_count ranges of pf_bytes (multiples of 16) at pf_base + i * pf_stride floats
+  const float* pf_base;
+  int pf_count, pf_bytes;
+  long long pf_stride;
 };
 
 // Tile widths used for each GEMM of the step (the weight layouts depend on them).

@@ -93,6 +93,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_arrive_expect_tx(&full[i], stage_tx);
       tma_load_2d(smem + i * C::kStageBytes + C::kABytes, &tmB, (kb0 + i) * kBK, n0, &full[i]);
     }
+    if (ep.pf_count > 0 && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0)
+      for (int i = 0; i < ep.pf_count; ++i) prefetch_l2(ep.pf_base + i * ep.pf_stride, ep.pf_bytes);
     pdl_wait();
     for (int i = 0; i < pre; ++i)
       tma_load_2d(smem + i * C::kStageBytes, &tmA, (kb0 + i) * kBK, m0, &full[i]);
