@@ -10,16 +10,22 @@
 
 namespace fva {
 
-// 64 bytes of one output row, straight from registers (16-byte stores): no
-// shared-memory staging, whose write and read-back would compete with the MMAs'
-// operand traffic for the SM's shared-memory bandwidth.
+// 32 bytes (one L2 sector) in one 256-bit store; dst 32-byte aligned.
+__device__ __forceinline__ void st_global_v8(void* dst, const uint4& a, const uint4& b) {
+  asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(dst), "r"(a.x),
+               "r"(a.y), "r"(a.z), "r"(a.w), "r"(b.x), "r"(b.y), "r"(b.z), "r"(b.w)
+               : "memory");
+}
+
+// 64 bytes of one output row, straight from registers as two 256-bit stores (each a
+// whole L2 sector; the 32 lanes of a warp write 32 different rows); dst 32-byte
+// aligned (every caller's row pieces start on 64-byte boundaries).  No shared-memory
+// staging, whose write and read-back would compete with the MMAs' operand traffic
+// for the SM's shared-memory bandwidth.
 __device__ __forceinline__ void store_row64(const uint4 (&u)[4], void* dst) {
   if (dst) {
-    uint4* d = reinterpret_cast<uint4*>(dst);
-    d[0] = u[0];
-    d[1] = u[1];
-    d[2] = u[2];
-    d[3] = u[3];
+    st_global_v8(dst, u[0], u[1]);
+    st_global_v8(reinterpret_cast<uint8_t*>(dst) + 32, u[2], u[3]);
   }
 }
 
