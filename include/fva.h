@@ -368,7 +368,7 @@ typedef enum fva_kernel_kind {
   FVA_K_FINAL = 10,          /* last gated residual + final FiLM RMSNorm (fp32 out)  */
   FVA_K_ATTN_MERGE = 11,     /* combination of the attention's key splits            */
   FVA_K_VELOCITY = 12,       /* out-projection + Euler + emit + roll + tail          */
-  FVA_K_BLOCK = 13,          /* reserved (no longer launched)                        */
+  FVA_K_PARAMS = 13,         /* the step's tau, dt, step index from the pinned ring   */
   FVA_K_COUNT = 14
 } fva_kernel_kind;
 

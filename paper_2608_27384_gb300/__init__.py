@@ -64,7 +64,7 @@ class fva_kernel_time(ctypes.Structure):
 
 KERNEL_KINDS = ["timestep_embed", "time_mlp", "film", "embed_norm", "qkv", "attention",
                 "out_proj", "resid_norm", "gate_up", "down", "final_norm", "attn_merge",
-                "velocity", "reserved_13"]
+                "velocity", "params"]
 
 EXPORTS = ["fva_create", "fva_destroy", "fva_num_weights", "fva_weight_shape",
            "fva_load_weights", "fva_set_prefix_kv", "fva_step", "fva_step_ex",

@@ -178,6 +178,9 @@ struct fva_handle {
   // per-step parameters: [tau BKmax | dt BKmax | step u64]
   float* params_dev = nullptr;
   float* params_host = nullptr;  // pinned ring [FVA_PARAM_RING][params_floats]
+  float* params_host_dev = nullptr;  // the ring's device address (mapped pinned memory)
+  int* ring_ctr = nullptr;  // device: slot the next step's fetch kernel reads
+  bool fetch_enqueued = false;  // enqueue_step queued the parameter fetch
   int params_floats = 0;
   cudaEvent_t ring_ev[FVA_PARAM_RING] = {};
   bool ring_used[FVA_PARAM_RING] = {};
@@ -462,6 +465,8 @@ static fva_status create_impl(const fva_config* cfg, fva_handle* h) {
   if ((st = dalloc(h, &h->params_dev, h->params_floats))) return st;
   CUDA_TRY(cudaMallocHost((void**)&h->params_host,
                           sizeof(float) * h->params_floats * FVA_PARAM_RING));
+  CUDA_TRY(cudaHostGetDevicePointer((void**)&h->params_host_dev, h->params_host, 0));
+  if ((st = dalloc(h, &h->ring_ctr, 1))) return st;
   CUDA_TRY(cudaMallocHost((void**)&h->err_host, sizeof(int)));
   *h->err_host = 0;
   for (auto& e : h->ring_ev) CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
@@ -940,6 +945,13 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   };
 
 
+  // ---- this step's tau, dt, step index and padding counts from its ring slot
+  mark(FVA_K_PARAMS, -1);
+  launch_fetch_params(h->params_host_dev, h->params_floats, FVA_PARAM_RING, h->ring_ctr,
+                      h->params_dev, s);
+  CUDA_TRY(cudaGetLastError());
+  h->fetch_enqueued = true;
+
   // ---- per-chunk FiLM condition and modulation (App. A.4); reused from the previous
   // step when the host saw identical noise levels (FVA_STEP_REUSE_FILM)
   // a projection with at least two tiles per SM and no K-split runs persistent, so
@@ -1175,6 +1187,20 @@ fva_status check_async_error(fva_handle* h, cudaStream_t s) {
   return FVA_OK;
 }
 
+// The step using ring slot `slot` is queued (its parameter fetch with it): the slot
+// may be written again once the stream has passed this point.
+void advance_ring(fva_handle* h, int slot, cudaStream_t s) {
+  h->ring_pos = (h->ring_pos + 1) % FVA_PARAM_RING;
+  if (cudaEventRecord(h->ring_ev[slot], s) == cudaSuccess) {
+    h->ring_used[slot] = true;
+  } else {
+    cudaGetLastError();
+    cudaStreamSynchronize(s);  // no event: the slot is free once the stream is idle
+    cudaGetLastError();
+    h->ring_used[slot] = false;
+  }
+}
+
 fva_status get_graph(fva_handle* h, int B, float* buffer, float* out, bool fresh, bool reuse_film,
                      cudaGraphExec_t* exec) {
   for (auto& g : h->graphs)
@@ -1264,9 +1290,10 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
   fva_status st = check_async_error(h, s);
   if (st != FVA_OK) return st;
 
-  // stage tau, dt and the step index through a pinned ring slot
+  // stage tau, dt and the step index in the next slot of the pinned ring; the
+  // step's first kernel reads that slot (its device-side counter follows the host's
+  // ring position: both advance once per queued step)
   const int slot = h->ring_pos;
-  h->ring_pos = (h->ring_pos + 1) % FVA_PARAM_RING;
   if (h->ring_used[slot]) CUDA_TRY(cudaEventSynchronize(h->ring_ev[slot]));
   float* ph = h->params_host + (size_t)slot * h->params_floats;
   for (int r = 0; r < batch; ++r)
@@ -1282,10 +1309,6 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
   int* pad = reinterpret_cast<int*>(ph + 2 * h->BKmax + 2);
   for (int r = 0; r < h->Bmax; ++r)
     pad[r] = (opts && opts->n_valid && r < batch) ? (h->K - opts->n_valid[r]) * h->H : 0;
-  CUDA_TRY(cudaMemcpyAsync(h->params_dev, ph, sizeof(float) * h->params_floats,
-                           cudaMemcpyHostToDevice, s));
-  CUDA_TRY(cudaEventRecord(h->ring_ev[slot], s));
-  h->ring_used[slot] = true;
 
   const bool fresh = opts && opts->fresh_noise;
   // the previous step's FiLM modulation is reused only for the same batch and
@@ -1326,6 +1349,7 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     prof->kind = h->prof_kind;
     prof->layer = h->prof_layer;
     CUDA_TRY(cudaGraphLaunch(h->prof_exec, s));
+    advance_ring(h, slot, s);
   } else if ((opts && opts->trace_layer >= 0) || (h->cfg.flags & FVA_FLAG_NO_GRAPH)) {
     StepTrace tr;
     tr.reuse_film = reuse_film;
@@ -1333,12 +1357,16 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
       tr.layer = opts->trace_layer;
       tr.out = opts->trace_out;
     }
-    if ((st = enqueue_step(h, batch, buffer, out_chunk, fresh, tr, s)) != FVA_OK) return st;
+    h->fetch_enqueued = false;
+    st = enqueue_step(h, batch, buffer, out_chunk, fresh, tr, s);
+    if (h->fetch_enqueued) advance_ring(h, slot, s);
+    if (st != FVA_OK) return st;
   } else {
     cudaGraphExec_t exec;
     if ((st = get_graph(h, batch, buffer, out_chunk, fresh, reuse_film, &exec)) != FVA_OK)
       return st;
     CUDA_TRY(cudaGraphLaunch(exec, s));
+    advance_ring(h, slot, s);
   }
   if (!reuse_film) {
     h->film_valid = true;

@@ -89,6 +89,12 @@ void launch_gather_action_kv(const void* kv_layer, bool act_bf16, const int* pre
 void launch_mask_table(const int* prefix_len, int B, int T, int H, int* key_limit,
                        cudaStream_t s);
 
+// The step's parameter block (tau, dt, step index, padding tokens: `floats` values)
+// from ring slot *ctr % ring of the pinned host ring `ring_host` (its device
+// address) into `dst`; then ++*ctr.  The first kernel of every step.
+void launch_fetch_params(const float* ring_host, int floats, int ring, int* ctr, float* dst,
+                         cudaStream_t s);
+
 // y = the bf16 GeGLU epilogue's GELU of x (fp32 in and out).
 void launch_geglu_gelu(const float* x, float* y, long long n, cudaStream_t s);
 

@@ -832,6 +832,31 @@ void launch_gemv_silu(const void* in, const void* w, const float* bias, void* ou
              K, tau, freq);
 }
 
+// ----------------------------------------------------------------------------
+// Per-step parameters.  The host writes each step's block into the next slot of a
+// pinned ring and launches the step; this kernel, the step's first, copies the
+// block of the slot its counter names into device memory and advances the counter
+// (one step at a time on the stream, so every step reads the slot its own call
+// filled).  No copy-engine transfer on the stream.
+// ----------------------------------------------------------------------------
+__global__ void fetch_params_kernel(const float* __restrict__ ring_host, int floats, int ring,
+                                    int* __restrict__ ctr, float* __restrict__ dst) {
+  __shared__ int slot;
+  pdl_trigger();
+  pdl_wait();
+  if (threadIdx.x == 0) slot = *ctr % ring;
+  __syncthreads();
+  const float* src = ring_host + (size_t)slot * floats;
+  for (int i = threadIdx.x; i < floats; i += blockDim.x) dst[i] = src[i];
+  __syncthreads();
+  if (threadIdx.x == 0) *ctr = (*ctr + 1) % ring;
+}
+
+void launch_fetch_params(const float* ring_host, int floats, int ring, int* ctr, float* dst,
+                         cudaStream_t s) {
+  launch_pdl(fetch_params_kernel, dim3(1), dim3(128), 0, s, ring_host, floats, ring, ctr, dst);
+}
+
 // The bf16 GeGLU epilogue's GELU on an fp32 array (introspection of its accuracy).
 __global__ void geglu_gelu_kernel(const float* __restrict__ x, float* __restrict__ y, long long n) {
   for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n;

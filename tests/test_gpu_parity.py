@@ -305,14 +305,15 @@ def test_step_profile_matches_step_and_counts_launches():
         np.testing.assert_array_equal(d_a.cpu().numpy(), d_b.cpu().numpy())
         kinds = [k for k, _, _ in recs]
         L = wl.n_layers
-        # 2 time-MLP layers (the first computes the timestep embedding itself), FiLM,
-        # embed+norm; per layer QKV, attention, split merge (prefix 600 + 200 keys:
-        # 13 query tiles of 13 key blocks in splits of 2; a cluster of 8 would leave
-        # its CTAs as many blocks, so the global form), O-projection, norm, gate/up,
-        # down, norm (last layer: final norm); velocity
+        # the parameter fetch, 2 time-MLP layers (the first computes the timestep
+        # embedding itself), FiLM, embed+norm; per layer QKV, attention, split merge
+        # (prefix 600 + 200 keys: 13 query tiles of 13 key blocks in splits of 2; a
+        # cluster of 8 would leave its CTAs as many blocks, so the global form),
+        # O-projection, norm, gate/up, down, norm (last layer: final norm); velocity
+        assert kinds[0] == "params" and kinds.count("params") == 1, kinds
         assert kinds.count("attention") == L and kinds.count("attn_merge") == L, kinds
         assert kinds[-1] == "velocity" and "timestep_embed" not in kinds
-        assert len(recs) == 4 + 8 * L + 1, kinds
+        assert len(recs) == 5 + 8 * L + 1, kinds
         assert kinds[-2] == "final_norm"
         assert all(us > 0 for _, _, us in recs)
     finally:
