@@ -945,10 +945,13 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   };
 
 
-  // ---- this step's tau, dt, step index and padding counts from its ring slot
+  // ---- this step's tau, dt, step index and padding counts from its ring slot (with
+  // the timestep embeddings when the time MLP runs as the GEMV)
+  const bool gemv = bf && BK <= 32;
   mark(FVA_K_PARAMS, -1);
   launch_fetch_params(h->params_host_dev, h->params_floats, FVA_PARAM_RING, h->ring_ctr,
-                      h->params_dev, s);
+                      h->params_dev, gemv && !tr.reuse_film ? h->temb : nullptr, BK, W,
+                      h->temb_freq, s);
   CUDA_TRY(cudaGetLastError());
   h->fetch_enqueued = true;
 
@@ -966,9 +969,8 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
   GemmEpi ep{};
   ep.err = h->err_dev;
   if (!tr.reuse_film) {
-    // a few rows (bf16): the first time-MLP GEMV computes the timestep embeddings
-    // itself; otherwise they are a kernel of their own
-    const bool gemv = bf && BK <= 32;
+    // a few rows (bf16): the parameter fetch wrote the timestep embeddings;
+    // otherwise they are a kernel of their own
     if (!gemv) {
       mark(FVA_K_TIMESTEP_EMBED, -1);
       launch_temb(h->tau_dev(), h->temb_freq, BK, W, h->temb, bf, s);
@@ -978,8 +980,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       // (the GEMV walks its rows 16 at a time)
       if (gemv) {
         mark(FVA_K_TIME_MLP, -1);
-        launch_gemv_silu(nullptr, h->w_t1, h->b_t1, h->t1, BK, W, W, s, h->tau_dev(),
-                         h->temb_freq);
+        launch_gemv_silu(h->temb, h->w_t1, h->b_t1, h->t1, BK, W, W, s);
         mark(FVA_K_TIME_MLP, -1);
         launch_gemv_silu(h->t1, h->w_t2, h->b_t2, h->cond, BK, W, W, s);
       } else {

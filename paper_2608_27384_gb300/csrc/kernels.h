@@ -68,13 +68,10 @@ void launch_velocity_euler(const StepDims& d, const float* yF, const float* w_ou
                            const unsigned long long* step_idx, cudaStream_t s);
 
 // out = silu(in W^T + bias), bf16 [M, K] x [N, K] -> bf16 [M, N]; K a multiple of 8.
-// With tau != nullptr the input rows are instead the timestep embeddings of tau[0..M)
-// (freq as for launch_temb; K = W), computed inside the kernel.
 // gemv_init sets the shared-memory limit for K (once per handle).
 cudaError_t gemv_init(int K);
 void launch_gemv_silu(const void* in, const void* w, const float* bias, void* out, int M, int N,
-                      int K, cudaStream_t s, const float* tau = nullptr,
-                      const float2* freq = nullptr);
+                      int K, cudaStream_t s);
 
 // (cos, sin) of position x frequency for RoPE, fp32 and rounded to fp16 pairs.
 void launch_rope_table(float2* table, uint32_t* table_h, int n_pos, int dh, float theta,
@@ -91,9 +88,11 @@ void launch_mask_table(const int* prefix_len, int B, int T, int H, int* key_limi
 
 // The step's parameter block (tau, dt, step index, padding tokens: `floats` values)
 // from ring slot *ctr % ring of the pinned host ring `ring_host` (its device
-// address) into `dst`; then ++*ctr.  The first kernel of every step.
+// address) into `dst`; then ++*ctr.  The first kernel of every step.  With temb
+// (bf16 [temb_rows, W]) it also writes the timestep embeddings of the block's first
+// temb_rows values (freq as for launch_temb).
 void launch_fetch_params(const float* ring_host, int floats, int ring, int* ctr, float* dst,
-                         cudaStream_t s);
+                         void* temb, int temb_rows, int W, const float2* freq, cudaStream_t s);
 
 // y = the bf16 GeGLU epilogue's GELU of x (fp32 in and out).
 void launch_geglu_gelu(const float* x, float* y, long long n, cudaStream_t s);

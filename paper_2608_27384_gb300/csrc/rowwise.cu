@@ -730,7 +730,7 @@ __device__ __forceinline__ int warp_sum16_index(int lane) {
 __global__ void __launch_bounds__(32 * kGemvWarps)
     gemv_silu_kernel(const bf16* __restrict__ in, const bf16* __restrict__ w,
                      const float* __restrict__ bias, bf16* __restrict__ out, int M, int N,
-                     int K, const float* __restrict__ tau, const float2* __restrict__ freq) {
+                     int K) {
   extern __shared__ __align__(16) uint4 sin4[];  // [16][K/8]
   __shared__ __align__(8) uint64_t bar;
   __shared__ float part[kGemvCols][kGemvRows];   // the upper K halves' sums
@@ -757,26 +757,12 @@ __global__ void __launch_bounds__(32 * kGemvWarps)
   for (int m0 = 0; m0 < M; m0 += kGemvRows) {
     const int mr = min(kGemvRows, M - m0);
     __syncthreads();
-    if (tau) {
-      // the input rows are the timestep embeddings of tau[m0 ..]: computed here (the
-      // same arithmetic as temb_kernel) instead of read back from global memory
-      bf16* sinb = reinterpret_cast<bf16*>(sin4);
-      const int half = K / 2;
-      for (int i = threadIdx.x; i < mr * half; i += blockDim.x) {
-        const int mm = i / half, j = i - mm * half;
-        const float2 sc = temb_sincos(tau[m0 + mm], freq[j]);
-        sinb[mm * K + j] = __float2bfloat16_rn(sc.x);
-        sinb[mm * K + half + j] = __float2bfloat16_rn(sc.y);
-      }
-      __syncthreads();
-    } else {
-      if (threadIdx.x == 0) {
-        mbar_arrive_expect_tx(&bar, (uint32_t)(mr * K * 2));
-        bulk_load(sin4, in + (size_t)m0 * K, (uint32_t)(mr * K * 2), &bar);
-      }
-      mbar_wait(&bar, phase, nullptr, 0);
-      phase ^= 1u;
+    if (threadIdx.x == 0) {
+      mbar_arrive_expect_tx(&bar, (uint32_t)(mr * K * 2));
+      bulk_load(sin4, in + (size_t)m0 * K, (uint32_t)(mr * K * 2), &bar);
     }
+    mbar_wait(&bar, phase, nullptr, 0);
+    phase ^= 1u;
     float acc[kGemvRows];
 #pragma unroll
     for (int mm = 0; mm < kGemvRows; ++mm) acc[mm] = 0.f;
@@ -825,11 +811,11 @@ cudaError_t gemv_init(int K) {
 }
 
 void launch_gemv_silu(const void* in, const void* w, const float* bias, void* out, int M, int N,
-                      int K, cudaStream_t s, const float* tau, const float2* freq) {
+                      int K, cudaStream_t s) {
   if (M <= 0) return;
   launch_pdl(gemv_silu_kernel, dim3((N + kGemvCols - 1) / kGemvCols), dim3(32 * kGemvWarps),
              (size_t)kGemvRows * K * 2, s, (const bf16*)in, (const bf16*)w, bias, (bf16*)out, M, N,
-             K, tau, freq);
+             K);
 }
 
 // ----------------------------------------------------------------------------
@@ -839,8 +825,14 @@ void launch_gemv_silu(const void* in, const void* w, const float* bias, void* ou
 // (one step at a time on the stream, so every step reads the slot its own call
 // filled).  No copy-engine transfer on the stream.
 // ----------------------------------------------------------------------------
-__global__ void fetch_params_kernel(const float* __restrict__ ring_host, int floats, int ring,
-                                    int* __restrict__ ctr, float* __restrict__ dst) {
+// With temb != nullptr it also writes the sinusoidal timestep embeddings of the
+// step's first temb_rows noise levels (the first values of the block), as
+// temb_kernel does, so that the time MLP reads them instead of every one of its CTAs
+// computing them.
+__global__ void __launch_bounds__(1024)
+    fetch_params_kernel(const float* __restrict__ ring_host, int floats, int ring,
+                        int* __restrict__ ctr, float* __restrict__ dst, bf16* __restrict__ temb,
+                        int temb_rows, int W, const float2* __restrict__ freq) {
   __shared__ int slot;
   pdl_trigger();
   pdl_wait();
@@ -848,13 +840,23 @@ __global__ void fetch_params_kernel(const float* __restrict__ ring_host, int flo
   __syncthreads();
   const float* src = ring_host + (size_t)slot * floats;
   for (int i = threadIdx.x; i < floats; i += blockDim.x) dst[i] = src[i];
+  if (temb) {
+    const int half = W / 2;
+    for (int i = threadIdx.x; i < temb_rows * half; i += blockDim.x) {
+      const int row = i / half, j = i - row * half;
+      const float2 sc = temb_sincos(src[row], freq[j]);
+      temb[(size_t)row * W + j] = __float2bfloat16_rn(sc.x);
+      temb[(size_t)row * W + half + j] = __float2bfloat16_rn(sc.y);
+    }
+  }
   __syncthreads();
   if (threadIdx.x == 0) *ctr = (*ctr + 1) % ring;
 }
 
 void launch_fetch_params(const float* ring_host, int floats, int ring, int* ctr, float* dst,
-                         cudaStream_t s) {
-  launch_pdl(fetch_params_kernel, dim3(1), dim3(128), 0, s, ring_host, floats, ring, ctr, dst);
+                         void* temb, int temb_rows, int W, const float2* freq, cudaStream_t s) {
+  launch_pdl(fetch_params_kernel, dim3(1), dim3(temb ? 1024 : 128), 0, s, ring_host, floats,
+             ring, ctr, dst, (bf16*)temb, temb_rows, W, freq);
 }
 
 // The bf16 GeGLU epilogue's GELU on an fp32 array (introspection of its accuracy).

@@ -305,8 +305,8 @@ def test_step_profile_matches_step_and_counts_launches():
         np.testing.assert_array_equal(d_a.cpu().numpy(), d_b.cpu().numpy())
         kinds = [k for k, _, _ in recs]
         L = wl.n_layers
-        # the parameter fetch, 2 time-MLP layers (the first computes the timestep
-        # embedding itself), FiLM, embed+norm; per layer QKV, attention, split merge
+        # the parameter fetch (which also writes the timestep embeddings), 2 time-MLP
+        # layers, FiLM, embed+norm; per layer QKV, attention, split merge
         # (prefix 600 + 200 keys: 13 query tiles of 13 key blocks in splits of 2; a
         # cluster of 8 would leave its CTAs as many blocks, so the global form),
         # O-projection, norm, gate/up, down, norm (last layer: final norm); velocity
