@@ -541,13 +541,16 @@ __global__ void __launch_bounds__(kVelThreads)
     mbar_arrive_expect_tx(&bar, (uint32_t)(sizeof(float) * (d.K + d.A) * wchunk));
     bulk_load(ws, w_out_t + (size_t)wbeg * d.A, (uint32_t)(sizeof(float) * wchunk * d.A), &bar);
   }
-  pdl_wait();
+  // this column of the buffer: written by the previous step's roll (earlier on the
+  // stream) and only read by this step's kernels before this one writes it, so it is
+  // read before the wait too
   const size_t slot = (size_t)d.H * d.A;
   const float* xcol = buffer + ((size_t)r * d.K * d.H + j) * d.A;  // + k*slot selects chunk k
   for (int i = threadIdx.x; i < KA; i += blockDim.x) {
     if (q == 0) xs[i] = xcol[(i / d.A) * slot + i % d.A];
     vs[i] = 0.f;
   }
+  pdl_wait();
   uint32_t phase = 0;
   for (int w0 = wbeg; w0 < wbeg + wq; w0 += wchunk) {
     __syncthreads();  // previous chunk consumed
