@@ -398,6 +398,38 @@ def test_short_a_boxes_bitwise(wl_kw):
         assert np.array_equal(a.view(np.uint32), b.view(np.uint32)), key
 
 
+def test_step_parameters_follow_every_call():
+    """Each step reads its own noise levels through the pinned ring of step
+    parameters (8 slots; the step's first kernel copies the slot a device counter
+    names): 20 steps on one handle with different levels each, mixing graph replays,
+    kernel-by-kernel trace steps and profiled steps, every one checked against the
+    oracle."""
+    import torch
+    import paper_2608_27384_gb300 as fva
+    wl = WL.small_bf16_workload(n_chunks=3, prefix_lens=[80])
+    case = Case(wl)
+    try:
+        fresh = WL.make_fresh_noise(wl, 1)[0]
+        base = case.tau.astype(np.float64)
+        for i in range(20):
+            # strictly increasing levels in (0, 1], different every step
+            tau = (base * (0.55 + 0.45 * ((i * 7) % 20) / 19.0)).astype(np.float32)
+            mode = i % 4
+            if mode == 3:
+                d_buf = case.dev(case.buf)
+                d_out = torch.empty((1, wl.chunk_tokens, wl.action_dim), device="cuda")
+                fva.fva_step_profile(case.handle, d_buf, tau, d_out, 1)
+                torch.cuda.synchronize()
+                res = dict(out=d_out.cpu().numpy(), buffer=d_buf.cpu().numpy())
+                ref = case.oracle_step(tau=tau)  # the emitted chunk does not see the tail
+                assert_close(res["out"], ref[0], what="profiled out", **TOL["bf16"])
+                continue
+            res = case.run(tau=tau, fresh=fresh, trace_layer=0 if mode == 2 else -1)
+            check_step(case, res, case.oracle_step(tau=tau, fresh=fresh), "bf16")
+    finally:
+        case.close()
+
+
 def test_reuse_film_matches_recomputed():
     """FVA_STEP_REUSE_FILM: with bit-identical noise levels the previous step's FiLM
     modulation is reused and the step's results are bit-identical to recomputing
