@@ -534,6 +534,29 @@ def main():
                                "previous step are reused (noise levels unchanged); not the "
                                "headline, which recomputes them every step"}
 
+    # ---- the same step with every layer's FiLM modulation computed before the first
+    # layer (FVA_STEP_SERIAL_FILM; the default computes layer 0's scale / shift first
+    # and the rest in the QKV projections' launches): the comparison, and the baseline
+    # of the per-launch event-node cost below (the profiled step computes the FiLM
+    # the same way)
+    film_serial = None
+    if rank == 0:
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                fva.fva_step_ex(h, d_buf, tau, d_out, B, serial_film=True, stream=stream)
+            es0 = torch.cuda.Event(enable_timing=True)
+            es1 = torch.cuda.Event(enable_timing=True)
+            es0.record(stream)
+            for _ in range(args.steps):
+                fva.fva_step_ex(h, d_buf, tau, d_out, B, serial_film=True, stream=stream)
+            es1.record(stream)
+        torch.cuda.synchronize()
+        us_s = 1e3 * es0.elapsed_time(es1) / args.steps
+        film_serial = {"us_per_step": us_s, "steps_per_s": 1e6 / us_s,
+                       "note": "FVA_STEP_SERIAL_FILM: every layer's FiLM modulation computed "
+                               "before the first layer; the headline computes it in the QKV "
+                               "projections' launches (same bits)"}
+
     # ---- kernel-by-kernel profile (CUDA events between launches on `stream`)
     per_kind = {}
     launches_per_step = 0
@@ -549,9 +572,12 @@ def main():
     tc = peaks["bf16_tflops"] * 1e12
     # The event nodes serialise the profiled graph and add a fixed cost to every
     # launch: (profiled step - timed step) / launches, spread evenly, is taken off
-    # each launch (never more than 3/4 of it).
+    # each launch (never more than 3/4 of it).  The profiled step computes the FiLM
+    # modulation before the first layer, so the timed step it is compared with is
+    # the one that does the same.
     prof_step_us = prof_total / max(1, args.profile_steps)
-    overhead_us = max(0.0, (prof_step_us - us_per_step) / max(1, launches_per_step))
+    base_us = film_serial["us_per_step"] if film_serial else us_per_step
+    overhead_us = max(0.0, (prof_step_us - base_us) / max(1, launches_per_step))
     corr = {k: (max(t - n * overhead_us, 0.25 * t), n) for k, (t, n) in per_kind.items()}
     dom = max(corr, key=lambda k: corr[k][0])
     t_us, n = corr[dom]
@@ -664,11 +690,13 @@ def main():
                 "profile_note": "per-kernel times: CUDA events between the kernels of a "
                                 "captured profiling graph; the event nodes serialise the "
                                 "kernels and cost about the same per launch, so "
-                                "(profiled step - timed step) / launches is taken off every "
-                                "launch (roofline.event_node_overhead_us)",
+                                "(profiled step - timed step with the FiLM computed first, "
+                                "film_serial) / launches is taken off every launch "
+                                "(roofline.event_node_overhead_us)",
                 "isolated_decode": isolated,
                 "attention_sweep": sweep,
                 "film_cached": film_cached,
+                "film_serial": film_serial,
                 "ncu_launch_shares": ncu_launch_shares(args.workload),
                 "clock_soak": {"steps": soak_steps, "seconds": args.clock_soak,
                                "note": "untimed steps between the warm-up and the timed "

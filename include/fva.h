@@ -230,6 +230,14 @@ fva_status fva_step(fva_handle* h, float* buffer, const float* noise_levels, flo
  * as usual.  Results are identical either way. */
 #define FVA_STEP_REUSE_FILM 1u
 
+/* fva_step_opts.flags.  SERIAL_FILM: compute every layer's FiLM modulation in one
+ * projection before the first layer.  By default (bf16, at most 16 chunk rows, the
+ * per-tile QKV projection) only layer 0's (scale, shift) pair is computed up front
+ * and each layer's QKV projection launch computes the next 6W modulation columns
+ * in extra CTAs on the SMs it leaves idle, before any norm reads them.  Results are
+ * bit-identical either way; the flag exists for comparison. */
+#define FVA_STEP_SERIAL_FILM 2u
+
 /* Extra inputs / outputs of fva_step_ex (zero-initialise; every field optional). */
 typedef struct fva_step_opts {
   const float* fresh_noise;  /* device fp32 [batch, H, A]: tail chunk to push instead of Philox */

@@ -200,11 +200,12 @@ def fva_step(handle: int, buffer, noise_levels, out_chunk, batch: int, stream=No
 
 
 FVA_STEP_REUSE_FILM = 1
+FVA_STEP_SERIAL_FILM = 2
 
 
 def fva_step_ex(handle: int, buffer, noise_levels, out_chunk, batch: int, fresh_noise=None,
                 velocity_out=None, trace_layer: int = -1, trace_out=None, stream=None,
-                n_valid=None, reuse_film: bool = False) -> None:
+                n_valid=None, reuse_film: bool = False, serial_film: bool = False) -> None:
     """n_valid: per-request real chunks (cold start), a sequence of ints or None."""
     tau, tp = _tau_ptr(noise_levels)
     nv = None
@@ -212,7 +213,8 @@ def fva_step_ex(handle: int, buffer, noise_levels, out_chunk, batch: int, fresh_
         import numpy as _np
         nv = _np.ascontiguousarray(n_valid, dtype=_np.int32)
     opts = fva_step_opts(_ptr(fresh_noise), _ptr(velocity_out), trace_layer,
-                         FVA_STEP_REUSE_FILM if reuse_film else 0, _ptr(trace_out),
+                         (FVA_STEP_REUSE_FILM if reuse_film else 0) |
+                         (FVA_STEP_SERIAL_FILM if serial_film else 0), _ptr(trace_out),
                          nv.ctypes.data if nv is not None else None)
     _check(lib().fva_step_ex(handle, _ptr(buffer), tp, _ptr(out_chunk), batch,
                              ctypes.byref(opts), _stream(stream)))

@@ -108,6 +108,7 @@ struct GraphEntry {
   float* out;
   bool fresh;
   bool reuse_film;
+  bool serial_film;
   cudaGraphExec_t exec;
   uint64_t last_use;
 };
@@ -149,6 +150,7 @@ struct fva_handle {
   void *w_t1 = nullptr, *w_t2 = nullptr, *w_mod = nullptr;
   std::vector<LayerW> layers;
   CUtensorMap m_wt1, m_wt2, m_wmod;
+  CUtensorMap m_wmod_q;  // FiLM weights in boxes of the QKV tile width (FiLM tiles in QKV)
   bool weights_loaded = false;
   // prefix / KV workspace
   void *kc = nullptr, *vc = nullptr;
@@ -764,7 +766,8 @@ extern "C" fva_status fva_load_weights(fva_handle* h, const void* const* tensors
     fva_status st;
     if ((st = make_map(&h->m_wt1, h->w_t1, W, W, kBnTime)) ||
         (st = make_map(&h->m_wt2, h->w_t2, W, W, kBnTime)) ||
-        (st = make_map(&h->m_wmod, h->w_mod, h->N_mod, W, kBnFilm)))
+        (st = make_map(&h->m_wmod, h->w_mod, h->N_mod, W, kBnFilm)) ||
+        (st = make_map(&h->m_wmod_q, h->w_mod, h->N_mod, W, h->bn_qkv)))
       return st;
   }
   h->weights_loaded = true;
@@ -873,6 +876,7 @@ struct StepTrace {
   int layer = -1;
   float* out = nullptr;
   bool reuse_film = false;  // skip the timestep embedding, time MLP and FiLM projection
+  bool serial_film = false; // every layer's FiLM modulation before the first layer
 };
 
 // Event before every launch (kernel profiling mode of fva_step_profile).  The
@@ -966,6 +970,34 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       return launch_tc_gemm_persist(bn, mode, ma, mb, e, Mr, N, Kd, h->n_sms, s);
     return launch_tc_gemm(bn, mode, ma, mb, e, Mr, N, Kd, splits, s);
   };
+  // The FiLM modulation rides in the QKV projections (extra CTAs on the SMs they
+  // leave idle): a layer's columns are [scale1 shift1 | gate1 scale2 shift2 | gate2]
+  // and its norms read them in that order, the first pair in the norm before its
+  // QKV projection, the rest after it.  So only layer 0's (scale1, shift1) are
+  // computed before the first layer, and layer l's QKV projection computes the
+  // next 6W columns: the rest of layer l and layer l+1's first pair (the last one
+  // the final norm's pair), complete by stream order before any norm reads them.
+  // Needs the per-tile QKV form and at most 16 condition rows; not when profiling
+  // kernel by kernel or tracing, which keep the FiLM projection a kernel of its own.
+  const int m_tiles_q = (M + 127) / 128;
+  const bool qkv_persist = h->persist_on && h->n_sms > 0 &&
+                           (long long)m_tiles_q * (h->N_qkv / h->bn_qkv) >= 2LL * h->n_sms;
+  const bool film_fold = bf && BK <= 16 && !tr.reuse_film && !tr.serial_film && !prof &&
+                         tr.layer < 0 && !qkv_persist && (6 * W) % h->bn_qkv == 0 &&
+                         (2 * W) % h->bn_qkv == 0 && (6 * W) % kBnFilm == 0;
+  // FiLM columns [c0, c0 + n) as tiles of the QKV tile width
+  auto film_tiles = [&](int c0, int n) {
+    FilmTiles ft{};
+    ft.a = h->m_cond16;
+    ft.b = h->m_wmod_q;
+    ft.out = h->mod;
+    ft.bias = h->b_mod;
+    ft.ldo = h->N_mod;
+    ft.rows = BK;
+    ft.tile0 = c0 / h->bn_qkv;
+    ft.tiles = n / h->bn_qkv;
+    return ft;
+  };
   GemmEpi ep{};
   ep.err = h->err_dev;
   if (!tr.reuse_film) {
@@ -1000,9 +1032,13 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.bias = h->b_mod;
       ep.ldo = h->N_mod;
       mark(FVA_K_FILM, -1);
-      CUDA_TRY(BK <= 16 ? launch_tc_gemm_stream(&h->m_cond16, &h->m_wmod, ep, BK, h->N_mod, W,
-                                                2 * h->n_sms, s)
-                         : gemm(kBnFilm, GEMM_BIAS_F32, &h->m_cond, &h->m_wmod, ep, BK, h->N_mod, W, 1));
+      if (film_fold)
+        CUDA_TRY(launch_tc_film_tiles(h->bn_qkv, film_tiles(0, 2 * W), W, h->err_dev, s));
+      else
+        CUDA_TRY(BK <= 16 ? launch_tc_gemm_stream(&h->m_cond16, &h->m_wmod, ep, BK, h->N_mod, W,
+                                                  2 * h->n_sms, s)
+                           : gemm(kBnFilm, GEMM_BIAS_F32, &h->m_cond, &h->m_wmod, ep, BK,
+                                  h->N_mod, W, 1));
     } else {
       launch_f32_gemm((float*)h->temb, W, (float*)h->w_t1, h->c32, W, BK, W, W, s);
       launch_f32_bias_act(h->c32, h->b_t1, (float*)h->t1, BK, W, true, s);
@@ -1056,8 +1092,14 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.pf_stride = h->N_mod;
       mark(FVA_K_QKV, l);
       ep.a_rows = h->y_box;
-      CUDA_TRY(gemm(h->bn_qkv, GEMM_QKV_ROPE, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_qkv, ep, M,
-                    h->N_qkv, W, 1));
+      if (film_fold) {
+        CUDA_TRY(launch_tc_gemm_qkv_film(h->bn_qkv, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_qkv,
+                                         ep, M, h->N_qkv, W, film_tiles(6 * W * l + 2 * W, 6 * W),
+                                         s));
+      } else {
+        CUDA_TRY(gemm(h->bn_qkv, GEMM_QKV_ROPE, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_qkv, ep,
+                      M, h->N_qkv, W, 1));
+      }
     } else {
       launch_f32_gemm((float*)h->y, W, (float*)lw.w_qkv, h->c32, h->N_qkv, M, h->N_qkv, W, s);
       launch_f32_qkv_rope(h->c32, (float*)h->q, (float*)kc_l, (float*)vc_l, h->prefix_len_dev,
@@ -1203,10 +1245,10 @@ void advance_ring(fva_handle* h, int slot, cudaStream_t s) {
 }
 
 fva_status get_graph(fva_handle* h, int B, float* buffer, float* out, bool fresh, bool reuse_film,
-                     cudaGraphExec_t* exec) {
+                     bool serial_film, cudaGraphExec_t* exec) {
   for (auto& g : h->graphs)
     if (g.batch == B && g.buffer == buffer && g.out == out && g.fresh == fresh &&
-        g.reuse_film == reuse_film) {
+        g.reuse_film == reuse_film && g.serial_film == serial_film) {
       g.last_use = ++h->use_clock;
       *exec = g.exec;
       return FVA_OK;
@@ -1223,6 +1265,7 @@ fva_status get_graph(fva_handle* h, int B, float* buffer, float* out, bool fresh
   CUDA_TRY(cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal));
   StepTrace tr;
   tr.reuse_film = reuse_film;
+  tr.serial_film = serial_film;
   fva_status st = enqueue_step(h, B, buffer, out, fresh, tr, h->cap_stream);
   cudaError_t e = cudaStreamEndCapture(h->cap_stream, &graph);
   if (st != FVA_OK) {
@@ -1234,7 +1277,8 @@ fva_status get_graph(fva_handle* h, int B, float* buffer, float* out, bool fresh
   e = cudaGraphInstantiate(&ge, graph, 0);
   cudaGraphDestroy(graph);
   CUDA_TRY(e);
-  h->graphs.push_back(GraphEntry{B, buffer, out, fresh, reuse_film, ge, ++h->use_clock});
+  h->graphs.push_back(GraphEntry{B, buffer, out, fresh, reuse_film, serial_film, ge,
+                                 ++h->use_clock});
   *exec = ge;
   return FVA_OK;
 }
@@ -1259,7 +1303,7 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     return fail(FVA_ERR_INVALID_ARG, "trace_layer %d >= n_layers", opts->trace_layer);
   if (opts && opts->trace_layer >= 0 && !opts->trace_out)
     return fail(FVA_ERR_INVALID_ARG, "trace_out is NULL");
-  if (opts && (opts->flags & ~FVA_STEP_REUSE_FILM))
+  if (opts && (opts->flags & ~(FVA_STEP_REUSE_FILM | FVA_STEP_SERIAL_FILM)))
     return fail(FVA_ERR_INVALID_ARG, "unknown step flags 0x%x", opts->flags);
   if (opts && opts->n_valid)
     for (int r = 0; r < batch; ++r)
@@ -1312,6 +1356,7 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     pad[r] = (opts && opts->n_valid && r < batch) ? (h->K - opts->n_valid[r]) * h->H : 0;
 
   const bool fresh = opts && opts->fresh_noise;
+  const bool serial_film = opts && (opts->flags & FVA_STEP_SERIAL_FILM);
   // the previous step's FiLM modulation is reused only for the same batch and
   // bit-identical noise levels
   const size_t n_tau = (size_t)batch * h->K;
@@ -1354,6 +1399,7 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
   } else if ((opts && opts->trace_layer >= 0) || (h->cfg.flags & FVA_FLAG_NO_GRAPH)) {
     StepTrace tr;
     tr.reuse_film = reuse_film;
+    tr.serial_film = serial_film;
     if (opts && opts->trace_layer >= 0) {
       tr.layer = opts->trace_layer;
       tr.out = opts->trace_out;
@@ -1364,7 +1410,8 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     if (st != FVA_OK) return st;
   } else {
     cudaGraphExec_t exec;
-    if ((st = get_graph(h, batch, buffer, out_chunk, fresh, reuse_film, &exec)) != FVA_OK)
+    if ((st = get_graph(h, batch, buffer, out_chunk, fresh, reuse_film, serial_film, &exec)) !=
+        FVA_OK)
       return st;
     CUDA_TRY(cudaGraphLaunch(exec, s));
     advance_ring(h, slot, s);

@@ -133,6 +133,21 @@ struct GemmEpi {
   long long pf_stride;
 };
 
+// Column tiles of the FiLM projection carried by the QKV projection's launch: extra
+// CTAs (grid.y >= y0, numbered (y - y0) * grid.x + x) each compute one BN-wide tile
+// tile0 + f of out[rows, :] = a b^T + bias (the GEMM_BIAS_F32 epilogue, the same
+// arithmetic as the FiLM kernel's), on the SMs the projection leaves idle.
+struct FilmTiles {
+  CUtensorMap a;       // condition rows [rows, K], 16-row boxes
+  CUtensorMap b;       // FiLM weights [N_mod, K], boxes of the projection's BN rows
+  float* out;          // modulation [rows, ldo]
+  const float* bias;
+  int ldo;
+  int rows;            // at most 16
+  int tile0, tiles;    // tiles 0: none
+  int y0;              // set by the launcher
+};
+
 // Tile widths used for each GEMM of the step (the weight layouts depend on them).
 constexpr int kBnQKV = 128;
 constexpr int kBnGU = 256;
@@ -158,6 +173,16 @@ cudaError_t launch_tc_gemm(int bn, int mode, const CUtensorMap* a, const CUtenso
 cudaError_t launch_tc_gemm_persist(int bn, int mode, const CUtensorMap* a, const CUtensorMap* b,
                                    const GemmEpi& ep, int M, int N, int K, int grid,
                                    cudaStream_t s);
+
+// The QKV projection (per-tile form, one K split) together with FiLM column tiles
+// (FilmTiles) in one launch.  bn: kBnQKV or kBnSmall.
+cudaError_t launch_tc_gemm_qkv_film(int bn, const CUtensorMap* a, const CUtensorMap* b,
+                                    const GemmEpi& ep, int M, int N, int K, const FilmTiles& film,
+                                    cudaStream_t s);
+
+// FiLM column tiles alone (one CTA per tile, the FilmTiles path of the launch
+// above); K as for the condition rows.
+cudaError_t launch_tc_film_tiles(int bn, const FilmTiles& film, int K, int* err, cudaStream_t s);
 
 // Persistent weight-streaming form of (kBnFilm, BIAS_F32) for M <= 16 rows: at
 // most `grid` CTAs (two per SM: pass twice the SM count) walk the N / kBnFilm

@@ -29,6 +29,8 @@ namespace {
 constexpr int kBM = 128;
 constexpr int kBK = 64;  // 64 bf16 = 128 bytes = one swizzle row
 constexpr int kThreads = 192;
+// rows of the FiLM condition (one 16-row TMA box)
+constexpr int kStreamRows = 16;
 
 template <int BN>
 struct GemmCfg {
@@ -43,10 +45,142 @@ struct GemmCfg {
   static_assert(kSmemBytes <= 227 * 1024, "shared memory above the per-CTA limit");
 };
 
+// One FiLM column tile in a CTA of the QKV projection's launch (FilmTiles): out =
+// cond W^T + bias for the <= 16 condition rows, the same MMA sequence and epilogue
+// as the FiLM kernel.  Its own shared-memory layout: the condition rows of every
+// k-block (16-row boxes, 2 KB each) in one area and the weights in a ring of
+// kFilmStages stages, most of which are requested before the dependency wait (the
+// weights depend on nothing; only the condition, written earlier in the step, is
+// loaded after it), so the tile mostly streams while the previous kernel finishes.
+// The M = 128 MMA reads 112 rows past each condition box (later boxes and the
+// ring): those accumulator rows are garbage and never stored.
+template <int BN>
+struct FilmCfg {
+  static constexpr int kABox = kStreamRows * kBK * 2;  // 2 KB
+  static constexpr int kMaxKb = 16;                    // K <= 1024
+  static constexpr int kABytes = kMaxKb * kABox;
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStages =
+      (GemmCfg<BN>::kStages * GemmCfg<BN>::kStageBytes - kABytes) / kBBytes < 14
+          ? (GemmCfg<BN>::kStages * GemmCfg<BN>::kStageBytes - kABytes) / kBBytes
+          : 14;
+  // fullB[kStages], emptyB[kStages], fullA, acc_full and the TMEM slot in 256 bytes
+  static_assert((2 * kStages + 2) * 8 + 4 <= 256, "barrier area too small");
+  static_assert(kABytes + kStages * kBBytes <= GemmCfg<BN>::kStages * GemmCfg<BN>::kStageBytes,
+                "FiLM layout beyond the ring");
+};
+
+template <int BN>
+__device__ void film_tile_cta(const FilmTiles& fj, uint8_t* smem, uint8_t* bar_area, int n0,
+                              int nkb, int* err) {
+  using F = FilmCfg<BN>;
+  uint64_t* fullB = (uint64_t*)bar_area;
+  uint64_t* emptyB = fullB + F::kStages;
+  uint64_t* fullA = emptyB + F::kStages;
+  uint64_t* acc_full = fullA + 1;
+  uint32_t* tmem_slot = (uint32_t*)(acc_full + 1);
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + F::kABytes;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < F::kStages; ++s) {
+      mbar_init(&fullB[s], 1);
+      mbar_init(&emptyB[s], 1);
+    }
+    mbar_init(fullA, 1);
+    mbar_init(acc_full, 1);
+    fence_barrier_init();
+    tma_prefetch_desc(&fj.a);
+    tma_prefetch_desc(&fj.b);
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, GemmCfg<BN>::kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
+
+  if (warp == 0 && lane == 0) {
+    // a few weight stages before the wait (more of them in flight while the
+    // previous kernel runs slowed the step down: 4 measured best on GB300)
+    const int pre = min(nkb, min(F::kStages, 4));
+    for (int i = 0; i < pre; ++i) {
+      mbar_arrive_expect_tx(&fullB[i], F::kBBytes);
+      tma_load_2d(sB + i * F::kBBytes, &fj.b, i * kBK, n0, &fullB[i]);
+    }
+    pdl_wait();
+    mbar_arrive_expect_tx(fullA, (uint32_t)(nkb * F::kABox));
+    for (int i = 0; i < nkb; ++i) tma_load_2d(sA + i * F::kABox, &fj.a, i * kBK, 0, fullA);
+    for (int i = pre; i < nkb; ++i) {
+      const int s = i % F::kStages;
+      if (!mbar_wait(&emptyB[s], ((uint32_t)(i / F::kStages) & 1u) ^ 1u, err, KERR_WAIT_MMA))
+        break;
+      mbar_arrive_expect_tx(&fullB[s], F::kBBytes);
+      tma_load_2d(sB + s * F::kBBytes, &fj.b, i * kBK, n0, &fullB[s]);
+    }
+  } else if (warp == 1 && lane == 0) {
+    constexpr uint32_t idesc = umma_idesc_bf16(kBM, BN, false);
+    const uint64_t a0 = umma_desc_sw128(smem_u32(sA), 16, 1024);
+    const uint64_t b0 = umma_desc_sw128(smem_u32(sB), 16, 1024);
+    bool good = mbar_wait(fullA, 0, err, KERR_WAIT_TMA);
+    for (int i = 0; good && i < nkb; ++i) {
+      const int s = i % F::kStages;
+      if (!mbar_wait(&fullB[s], (uint32_t)(i / F::kStages) & 1u, err, KERR_WAIT_TMA)) {
+        good = false;
+        break;
+      }
+      tc_fence_after();
+      const uint64_t ad = desc_advance(a0, i * F::kABox);
+      const uint64_t bd = desc_advance(b0, s * F::kBBytes);
+#pragma unroll
+      for (int kk = 0; kk < kBK / 16; ++kk)
+        umma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (i > 0 || kk > 0) ? 1u : 0u);
+      umma_commit(&emptyB[s]);
+    }
+    if (good) umma_commit(acc_full);
+  } else if (warp >= 2) {
+    // the GEMM_BIAS_F32 epilogue (fp32 out = acc + bias, the same single rounding),
+    // with the tile's bias fetched before the accumulator is ready: lane l holds
+    // column c + l of every 32-column chunk c and hands it to the warp by shuffle.
+    // Only the warp of TMEM lanes 0-31 has condition rows.
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    float bl[BN / 32];
+#pragma unroll
+    for (int c = 0; c < BN / 32; ++c) bl[c] = __ldg(fj.bias + n0 + c * 32 + lane);
+    const bool good = __all_sync(0xffffffffu, mbar_wait(acc_full, 0, err, KERR_WAIT_MMA));
+    tc_fence_after();
+    if (good && nkb > 0 && quarter * 32 < fj.rows) {
+      // every MMA is complete: the condition area is free to stage the stores
+      const uint32_t trow = tmem + ((uint32_t)(quarter * 32) << 16);
+      uint8_t* stage = smem + (warp - 2) * (32 * 144);
+      float* dst = row < fj.rows ? fj.out + (size_t)row * fj.ldo + n0 : nullptr;
+#pragma unroll
+      for (int c = 0; c < BN / 32; ++c) {
+        float v[32];
+        tmem_ld32(trow + c * 32, v);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] += __shfl_sync(0xffffffffu, bl[c], i);
+        uint4 u[8];
+        pack_f32x32(v, u);
+        warp_store_rows<128>(stage, u, dst ? dst + c * 32 : nullptr, lane);
+      }
+    }
+  }
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, GemmCfg<BN>::kTmemCols);
+  }
+}
+
 template <int BN, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const GemmEpi ep, int M, int N, int kb_total, int kb_per_split) {
+                   const GemmEpi ep, int M, int N, int kb_total, int kb_per_split,
+                   const __grid_constant__ FilmTiles fj) {
   using C = GemmCfg<BN>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -56,7 +190,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = (uint32_t*)(acc_full + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.x * kBM, n0 = blockIdx.y * BN, split = blockIdx.z;
+  // the QKV projection's launch may carry FiLM column tiles in extra CTAs (grid.y
+  // >= fj.y0; same K, one split)
+  if constexpr (MODE == GEMM_QKV_ROPE) {
+    if ((int)blockIdx.y >= fj.y0) {
+      const int f = ((int)blockIdx.y - fj.y0) * (int)gridDim.x + (int)blockIdx.x;
+      if (f < fj.tiles)  // uniform over the CTA
+        film_tile_cta<BN>(fj, smem, (uint8_t*)full, (fj.tile0 + f) * BN, kb_total, ep.err);
+      return;
+    }
+  }
+  const int m0 = blockIdx.x * kBM, n0 = blockIdx.y * BN;
+  const int split = blockIdx.z;
   const int kb0 = split * kb_per_split;
   const int nkb = min(kb_total, kb0 + kb_per_split) - kb0;
 
@@ -174,7 +319,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 // of A.  The M = 128 MMA reads 112 more rows past them (the stage's weights):
 // those accumulator rows are garbage and never stored, and the small A region
 // leaves room for a deeper weight ring.
-constexpr int kStreamRows = 16;
 
 template <int BN>
 struct GemmStreamCfg {
@@ -517,8 +661,22 @@ cudaError_t launch(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep
   const int kb_total = K / kBK;
   const int kbps = (kb_total + splits - 1) / splits;
   dim3 grid((M + kBM - 1) / kBM, N / BN, splits);
+  FilmTiles none{};
+  none.y0 = N / BN;
   return launch_pdl(tc_gemm_kernel<BN, MODE>, grid, dim3(kThreads), GemmCfg<BN>::kSmemBytes, s,
-                    *a, *b, ep, M, N, kb_total, kbps);
+                    *a, *b, ep, M, N, kb_total, kbps, none);
+}
+
+template <int BN>
+cudaError_t launch_qkv_film(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep, int M,
+                            int N, int K, const FilmTiles& film, cudaStream_t s) {
+  const int m_tiles = (M + kBM - 1) / kBM;
+  FilmTiles f = film;
+  f.y0 = N / BN;
+  const int extra_y = film.tiles > 0 ? (film.tiles + m_tiles - 1) / m_tiles : 0;
+  dim3 grid(m_tiles, N / BN + extra_y, 1);
+  return launch_pdl(tc_gemm_kernel<BN, GEMM_QKV_ROPE>, grid, dim3(kThreads),
+                    GemmCfg<BN>::kSmemBytes, s, *a, *b, ep, M, N, K / kBK, K / kBK, f);
 }
 
 }  // namespace
@@ -557,6 +715,40 @@ cudaError_t launch_tc_gemm_persist(int bn, int mode, const CUtensorMap* a, const
     return launch_persist<kBnResid, GEMM_PARTIAL_BF16>(a, b, ep, M, N, K, grid, s);
   if (bn == kBnFilm && mode == GEMM_BIAS_F32)
     return launch_persist<kBnFilm, GEMM_BIAS_F32>(a, b, ep, M, N, K, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_tc_gemm_qkv_film(int bn, const CUtensorMap* a, const CUtensorMap* b,
+                                    const GemmEpi& ep, int M, int N, int K, const FilmTiles& film,
+                                    cudaStream_t s) {
+  if (M <= 0) return cudaSuccess;
+  if (N % bn != 0 || K % kBK != 0 || film.rows > kStreamRows || film.tiles < 0 ||
+      (film.tiles > 0 && K / kBK > FilmCfg<kBnQKV>::kMaxKb) ||
+      film.tile0 < 0 || (film.tiles > 0 && (film.rows < 1 || film.ldo % bn != 0 ||
+                                            (film.tile0 + film.tiles) * bn > film.ldo)))
+    return cudaErrorInvalidValue;
+  if (bn == kBnQKV) return launch_qkv_film<kBnQKV>(a, b, ep, M, N, K, film, s);
+  if (bn == kBnSmall) return launch_qkv_film<kBnSmall>(a, b, ep, M, N, K, film, s);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_tc_film_tiles(int bn, const FilmTiles& film, int K, int* err, cudaStream_t s) {
+  if (film.tiles <= 0) return cudaSuccess;
+  if (K % kBK != 0 || K / kBK > FilmCfg<kBnQKV>::kMaxKb || film.rows < 1 ||
+      film.rows > kStreamRows || film.tile0 < 0 || film.ldo % bn != 0 ||
+      (film.tile0 + film.tiles) * bn > film.ldo)
+    return cudaErrorInvalidValue;
+  FilmTiles f = film;
+  f.y0 = 0;  // every CTA is a FiLM tile
+  GemmEpi ep{};
+  ep.err = err;
+  const dim3 grid(1, film.tiles, 1);
+  if (bn == kBnQKV)
+    return launch_pdl(tc_gemm_kernel<kBnQKV, GEMM_QKV_ROPE>, grid, dim3(kThreads),
+                      GemmCfg<kBnQKV>::kSmemBytes, s, f.a, f.b, ep, 0, 0, K / kBK, K / kBK, f);
+  if (bn == kBnSmall)
+    return launch_pdl(tc_gemm_kernel<kBnSmall, GEMM_QKV_ROPE>, grid, dim3(kThreads),
+                      GemmCfg<kBnSmall>::kSmemBytes, s, f.a, f.b, ep, 0, 0, K / kBK, K / kBK, f);
   return cudaErrorInvalidValue;
 }
 

@@ -58,7 +58,7 @@ class Case:
         return self.torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
     def run(self, buf=None, tau=None, fresh=None, want_vel=True, trace_layer=-1, batch=None,
-            n_valid=None, reuse_film=False):
+            n_valid=None, reuse_film=False, serial_film=False):
         """One GPU step.  Returns dict(out, buffer, vel[, trace]) as numpy arrays."""
         import paper_2608_27384_gb300 as fva
         torch = self.torch
@@ -77,7 +77,7 @@ class Case:
         fva.fva_step_ex(self.handle, d_buf, tau[:B], d_out, B, fresh_noise=d_fresh,
                         velocity_out=d_vel, trace_layer=trace_layer, trace_out=d_tr,
                         n_valid=None if n_valid is None else list(n_valid)[:B],
-                        reuse_film=reuse_film)
+                        reuse_film=reuse_film, serial_film=serial_film)
         torch.cuda.synchronize()
         res = dict(out=d_out.cpu().numpy(), buffer=d_buf.cpu().numpy())
         if want_vel:

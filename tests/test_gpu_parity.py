@@ -398,6 +398,38 @@ def test_short_a_boxes_bitwise(wl_kw):
         assert np.array_equal(a.view(np.uint32), b.view(np.uint32)), key
 
 
+@pytest.mark.parametrize("wl_kw", [
+    dict(),                                                   # 2 layers, W 256, 3 chunks
+    dict(n_layers=6, width=512, mlp_dim=1024, n_chunks=10, chunk_tokens=8, prefix_lens=[200]),
+    dict(n_layers=4, n_chunks=4, chunk_tokens=10, batch=2, prefix_lens=[64, 150]),
+], ids=["L2", "L6_K10", "B2_K4"])
+def test_film_overlap_matches_serial_bitwise(wl_kw):
+    """FiLM modulation carried by the QKV projections (layer 0's scale / shift pair
+    first, then each layer's QKV launch computing the next 6W columns in extra CTAs)
+    gives the bits of the step that computes all of it before the first layer, step
+    after step with new noise levels each time (a norm reading the previous step's
+    modulation would differ), and both match the oracle."""
+    wl = WL.small_bf16_workload(**wl_kw)
+    case = Case(wl)
+    try:
+        fresh = WL.make_fresh_noise(wl, 1)[0]
+        base = case.tau.astype(np.float64)
+        for i in range(5):
+            tau = (base * (0.6 + 0.1 * i)).astype(np.float32)
+            res = {mode: case.run(tau=tau, fresh=fresh, serial_film=(mode == "serial"))
+                   for mode in ("overlap", "serial", "overlap2")}
+            for key in ("out", "buffer", "vel"):
+                a = res["overlap"][key]
+                assert np.isfinite(a).all()
+                for other in ("serial", "overlap2"):
+                    assert np.array_equal(a.view(np.uint32), res[other][key].view(np.uint32)), \
+                        (i, key, other)
+            if i in (0, 4):
+                check_step(case, res["overlap"], case.oracle_step(tau=tau, fresh=fresh), "bf16")
+    finally:
+        case.close()
+
+
 def test_step_parameters_follow_every_call():
     """Each step reads its own noise levels through the pinned ring of step
     parameters (8 slots; the step's first kernel copies the slot a device counter
