@@ -150,7 +150,7 @@ struct fva_handle {
   void *w_t1 = nullptr, *w_t2 = nullptr, *w_mod = nullptr;
   std::vector<LayerW> layers;
   CUtensorMap m_wt1, m_wt2, m_wmod;
-  CUtensorMap m_wmod_q;  // FiLM weights in boxes of the QKV tile width (FiLM tiles in QKV)
+  CUtensorMap m_wmod_q;  // FiLM weights in kFilmTile-row boxes (FiLM tiles in projections)
   bool weights_loaded = false;
   // prefix / KV workspace
   void *kc = nullptr, *vc = nullptr;
@@ -767,7 +767,7 @@ extern "C" fva_status fva_load_weights(fva_handle* h, const void* const* tensors
     if ((st = make_map(&h->m_wt1, h->w_t1, W, W, kBnTime)) ||
         (st = make_map(&h->m_wt2, h->w_t2, W, W, kBnTime)) ||
         (st = make_map(&h->m_wmod, h->w_mod, h->N_mod, W, kBnFilm)) ||
-        (st = make_map(&h->m_wmod_q, h->w_mod, h->N_mod, W, h->bn_qkv)))
+        (st = make_map(&h->m_wmod_q, h->w_mod, h->N_mod, W, kFilmTile)))
       return st;
   }
   h->weights_loaded = true;
@@ -970,22 +970,34 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       return launch_tc_gemm_persist(bn, mode, ma, mb, e, Mr, N, Kd, h->n_sms, s);
     return launch_tc_gemm(bn, mode, ma, mb, e, Mr, N, Kd, splits, s);
   };
-  // The FiLM modulation rides in the QKV projections (extra CTAs on the SMs they
-  // leave idle): a layer's columns are [scale1 shift1 | gate1 scale2 shift2 | gate2]
-  // and its norms read them in that order, the first pair in the norm before its
-  // QKV projection, the rest after it.  So only layer 0's (scale1, shift1) are
-  // computed before the first layer, and layer l's QKV projection computes the
-  // next 6W columns: the rest of layer l and layer l+1's first pair (the last one
-  // the final norm's pair), complete by stream order before any norm reads them.
-  // Needs the per-tile QKV form and at most 16 condition rows; not when profiling
-  // kernel by kernel or tracing, which keep the FiLM projection a kernel of its own.
+  // The FiLM modulation rides in the QKV and gate/up projections' launches (extra
+  // CTAs of kFilmTile columns on the SMs they leave idle): a layer's columns are
+  // [scale1 shift1 | gate1 scale2 shift2 | gate2] and its norms read them in that
+  // order, the first pair in the norm before its QKV projection, the next three
+  // after its attention, the last after its MLP.  So only layer 0's (scale1,
+  // shift1) are computed before the first layer, and layer l's launches compute
+  // the next 6W columns: its QKV launch at least (gate1, scale2, shift2) and as many
+  // more as it has idle SMs for, its gate/up launch the rest (gate2 and layer l+1's
+  // first pair, the last layer's the final norm's pair), each complete by stream
+  // order before a norm reads it.  Needs the per-tile QKV form, at most 16
+  // condition rows and W <= 1024; not when profiling kernel by kernel or tracing,
+  // which keep the FiLM projection a kernel of its own.
   const int m_tiles_q = (M + 127) / 128;
-  const bool qkv_persist = h->persist_on && h->n_sms > 0 &&
-                           (long long)m_tiles_q * (h->N_qkv / h->bn_qkv) >= 2LL * h->n_sms;
+  const int qkv_ctas = m_tiles_q * (h->N_qkv / h->bn_qkv);
+  const int gu_ctas = m_tiles_q * (2 * F / h->bn_gu);
+  const bool qkv_persist = h->persist_on && h->n_sms > 0 && qkv_ctas >= 2 * h->n_sms;
+  const bool gu_persist = h->persist_on && h->n_sms > 0 && gu_ctas >= 2 * h->n_sms;
   const bool film_fold = bf && BK <= 16 && !tr.reuse_film && !tr.serial_film && !prof &&
-                         tr.layer < 0 && !qkv_persist && (6 * W) % h->bn_qkv == 0 &&
-                         (2 * W) % h->bn_qkv == 0 && (6 * W) % kBnFilm == 0;
-  // FiLM columns [c0, c0 + n) as tiles of the QKV tile width
+                         tr.layer < 0 && !qkv_persist && W % kFilmTile == 0 && W <= 1024;
+  const int film_group = 6 * W / kFilmTile;  // tiles computed by each layer's launches
+  int film_gu = 0;                           // of which in the gate/up launch
+  if (film_fold && !gu_persist) {
+    const int film_q_min = 3 * W / kFilmTile;
+    const int q = std::max(film_q_min, std::min(film_group, h->n_sms - qkv_ctas));
+    film_gu = std::min(film_group - q, std::max(0, h->n_sms - gu_ctas));
+  }
+  const int film_q = film_group - film_gu;
+  // FiLM columns [c0, c0 + n) as kFilmTile-wide tiles
   auto film_tiles = [&](int c0, int n) {
     FilmTiles ft{};
     ft.a = h->m_cond16;
@@ -994,8 +1006,8 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     ft.bias = h->b_mod;
     ft.ldo = h->N_mod;
     ft.rows = BK;
-    ft.tile0 = c0 / h->bn_qkv;
-    ft.tiles = n / h->bn_qkv;
+    ft.tile0 = c0 / kFilmTile;
+    ft.tiles = n / kFilmTile;
     return ft;
   };
   GemmEpi ep{};
@@ -1033,7 +1045,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.ldo = h->N_mod;
       mark(FVA_K_FILM, -1);
       if (film_fold)
-        CUDA_TRY(launch_tc_film_tiles(h->bn_qkv, film_tiles(0, 2 * W), W, h->err_dev, s));
+        CUDA_TRY(launch_tc_film_tiles(film_tiles(0, 2 * W), W, h->err_dev, s));
       else
         CUDA_TRY(BK <= 16 ? launch_tc_gemm_stream(&h->m_cond16, &h->m_wmod, ep, BK, h->N_mod, W,
                                                   2 * h->n_sms, s)
@@ -1093,9 +1105,9 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       mark(FVA_K_QKV, l);
       ep.a_rows = h->y_box;
       if (film_fold) {
-        CUDA_TRY(launch_tc_gemm_qkv_film(h->bn_qkv, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_qkv,
-                                         ep, M, h->N_qkv, W, film_tiles(6 * W * l + 2 * W, 6 * W),
-                                         s));
+        CUDA_TRY(launch_tc_gemm_film(h->bn_qkv, GEMM_QKV_ROPE, h->y_box ? &h->m_ybox : &h->m_y,
+                                     &lw.m_qkv, ep, M, h->N_qkv, W,
+                                     film_tiles(6 * W * l + 2 * W, film_q * kFilmTile), s));
       } else {
         CUDA_TRY(gemm(h->bn_qkv, GEMM_QKV_ROPE, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_qkv, ep,
                       M, h->N_qkv, W, 1));
@@ -1169,8 +1181,13 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.ldo = F;
       mark(FVA_K_GATE_UP, l);
       ep.a_rows = h->y_box;
-      CUDA_TRY(gemm(h->bn_gu, GEMM_GEGLU, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_gu, ep, M, 2 * F,
-                    W, 1));
+      if (film_fold && film_gu > 0)
+        CUDA_TRY(launch_tc_gemm_film(
+            h->bn_gu, GEMM_GEGLU, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_gu, ep, M, 2 * F, W,
+            film_tiles(6 * W * l + 2 * W + film_q * kFilmTile, film_gu * kFilmTile), s));
+      else
+        CUDA_TRY(gemm(h->bn_gu, GEMM_GEGLU, h->y_box ? &h->m_ybox : &h->m_y, &lw.m_gu, ep, M,
+                      2 * F, W, 1));
       ep.a_rows = 0;
       ep.out = h->part;
       ep.ldo = W;

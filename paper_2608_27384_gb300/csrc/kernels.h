@@ -133,13 +133,15 @@ struct GemmEpi {
   long long pf_stride;
 };
 
-// Column tiles of the FiLM projection carried by the QKV projection's launch: extra
-// CTAs (grid.y >= y0, numbered (y - y0) * grid.x + x) each compute one BN-wide tile
-// tile0 + f of out[rows, :] = a b^T + bias (the GEMM_BIAS_F32 epilogue, the same
-// arithmetic as the FiLM kernel's), on the SMs the projection leaves idle.
+// Column tiles of the FiLM projection carried by the QKV or gate/up projection's
+// launch: extra CTAs (grid.y >= y0, numbered (y - y0) * grid.x + x) each compute one
+// kFilmTile-wide tile tile0 + f of out[rows, :] = a b^T + bias (the GEMM_BIAS_F32
+// epilogue, the same arithmetic as the FiLM kernel's), on the SMs the projection
+// leaves idle.
+constexpr int kFilmTile = 64;
 struct FilmTiles {
   CUtensorMap a;       // condition rows [rows, K], 16-row boxes
-  CUtensorMap b;       // FiLM weights [N_mod, K], boxes of the projection's BN rows
+  CUtensorMap b;       // FiLM weights [N_mod, K], kFilmTile-row boxes
   float* out;          // modulation [rows, ldo]
   const float* bias;
   int ldo;
@@ -174,15 +176,15 @@ cudaError_t launch_tc_gemm_persist(int bn, int mode, const CUtensorMap* a, const
                                    const GemmEpi& ep, int M, int N, int K, int grid,
                                    cudaStream_t s);
 
-// The QKV projection (per-tile form, one K split) together with FiLM column tiles
-// (FilmTiles) in one launch.  bn: kBnQKV or kBnSmall.
-cudaError_t launch_tc_gemm_qkv_film(int bn, const CUtensorMap* a, const CUtensorMap* b,
-                                    const GemmEpi& ep, int M, int N, int K, const FilmTiles& film,
-                                    cudaStream_t s);
+// A QKV (GEMM_QKV_ROPE) or gate/up (GEMM_GEGLU) projection, per-tile form with one
+// K split, together with FiLM column tiles (FilmTiles) in one launch.
+cudaError_t launch_tc_gemm_film(int bn, int mode, const CUtensorMap* a, const CUtensorMap* b,
+                                const GemmEpi& ep, int M, int N, int K, const FilmTiles& film,
+                                cudaStream_t s);
 
 // FiLM column tiles alone (one CTA per tile, the FilmTiles path of the launch
 // above); K as for the condition rows.
-cudaError_t launch_tc_film_tiles(int bn, const FilmTiles& film, int K, int* err, cudaStream_t s);
+cudaError_t launch_tc_film_tiles(const FilmTiles& film, int K, int* err, cudaStream_t s);
 
 // Persistent weight-streaming form of (kBnFilm, BIAS_F32) for M <= 16 rows: at
 // most `grid` CTAs (two per SM: pass twice the SM count) walk the N / kBnFilm

@@ -45,35 +45,36 @@ struct GemmCfg {
   static_assert(kSmemBytes <= 227 * 1024, "shared memory above the per-CTA limit");
 };
 
-// One FiLM column tile in a CTA of the QKV projection's launch (FilmTiles): out =
-// cond W^T + bias for the <= 16 condition rows, the same MMA sequence and epilogue
-// as the FiLM kernel.  Its own shared-memory layout: the condition rows of every
-// k-block (16-row boxes, 2 KB each) in one area and the weights in a ring of
-// kFilmStages stages, most of which are requested before the dependency wait (the
-// weights depend on nothing; only the condition, written earlier in the step, is
-// loaded after it), so the tile mostly streams while the previous kernel finishes.
-// The M = 128 MMA reads 112 rows past each condition box (later boxes and the
-// ring): those accumulator rows are garbage and never stored.
-template <int BN>
+// One FiLM column tile (kFilmTile wide) in a CTA of a projection's launch
+// (FilmTiles): out = cond W^T + bias for the <= 16 condition rows, the same MMA
+// sequence and epilogue as the FiLM kernel.  Its own layout of the host kernel's
+// ring (kRingBytes): the condition rows of every k-block (16-row boxes, 2 KB each)
+// in one area and the weights in a ring of up to 14 stages, a few of which are
+// requested before the dependency wait (the weights depend on nothing; only the
+// condition, written earlier in the step, is loaded after it).  The M = 128 MMA
+// reads 112 rows past each condition box (later boxes and the ring): those
+// accumulator rows are garbage and never stored.
+constexpr int kFilmMaxKb = 16;  // K <= 1024
+
+template <int kRingBytes>
 struct FilmCfg {
   static constexpr int kABox = kStreamRows * kBK * 2;  // 2 KB
-  static constexpr int kMaxKb = 16;                    // K <= 1024
+  static constexpr int kMaxKb = kFilmMaxKb;
   static constexpr int kABytes = kMaxKb * kABox;
-  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kBBytes = kFilmTile * kBK * 2;
   static constexpr int kStages =
-      (GemmCfg<BN>::kStages * GemmCfg<BN>::kStageBytes - kABytes) / kBBytes < 14
-          ? (GemmCfg<BN>::kStages * GemmCfg<BN>::kStageBytes - kABytes) / kBBytes
-          : 14;
+      (kRingBytes - kABytes) / kBBytes < 14 ? (kRingBytes - kABytes) / kBBytes : 14;
   // fullB[kStages], emptyB[kStages], fullA, acc_full and the TMEM slot in 256 bytes
   static_assert((2 * kStages + 2) * 8 + 4 <= 256, "barrier area too small");
-  static_assert(kABytes + kStages * kBBytes <= GemmCfg<BN>::kStages * GemmCfg<BN>::kStageBytes,
+  static_assert(kStages >= 4 && kABytes + kStages * kBBytes <= kRingBytes,
                 "FiLM layout beyond the ring");
 };
 
-template <int BN>
+template <int kRingBytes>
 __device__ void film_tile_cta(const FilmTiles& fj, uint8_t* smem, uint8_t* bar_area, int n0,
                               int nkb, int* err) {
-  using F = FilmCfg<BN>;
+  using F = FilmCfg<kRingBytes>;
+  constexpr int BN = kFilmTile;
   uint64_t* fullB = (uint64_t*)bar_area;
   uint64_t* emptyB = fullB + F::kStages;
   uint64_t* fullA = emptyB + F::kStages;
@@ -93,7 +94,7 @@ __device__ void film_tile_cta(const FilmTiles& fj, uint8_t* smem, uint8_t* bar_a
     tma_prefetch_desc(&fj.a);
     tma_prefetch_desc(&fj.b);
   }
-  if (warp == 1) tmem_alloc(tmem_slot, GemmCfg<BN>::kTmemCols);
+  if (warp == 1) tmem_alloc(tmem_slot, BN);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -172,7 +173,7 @@ __device__ void film_tile_cta(const FilmTiles& fj, uint8_t* smem, uint8_t* bar_a
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, GemmCfg<BN>::kTmemCols);
+    tmem_dealloc(tmem, BN);
   }
 }
 
@@ -190,13 +191,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = (uint32_t*)(acc_full + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  // the QKV projection's launch may carry FiLM column tiles in extra CTAs (grid.y
-  // >= fj.y0; same K, one split)
-  if constexpr (MODE == GEMM_QKV_ROPE) {
+  // the QKV and gate/up projections' launches may carry FiLM column tiles in extra
+  // CTAs (grid.y >= fj.y0; same K, one split)
+  if constexpr (MODE == GEMM_QKV_ROPE || MODE == GEMM_GEGLU) {
     if ((int)blockIdx.y >= fj.y0) {
       const int f = ((int)blockIdx.y - fj.y0) * (int)gridDim.x + (int)blockIdx.x;
       if (f < fj.tiles)  // uniform over the CTA
-        film_tile_cta<BN>(fj, smem, (uint8_t*)full, (fj.tile0 + f) * BN, kb_total, ep.err);
+        film_tile_cta<C::kStages * C::kStageBytes>(fj, smem, (uint8_t*)full,
+                                                   (fj.tile0 + f) * kFilmTile, kb_total, ep.err);
       return;
     }
   }
@@ -667,16 +669,23 @@ cudaError_t launch(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep
                     *a, *b, ep, M, N, kb_total, kbps, none);
 }
 
-template <int BN>
-cudaError_t launch_qkv_film(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep, int M,
-                            int N, int K, const FilmTiles& film, cudaStream_t s) {
+template <int BN, int MODE>
+cudaError_t launch_film(const CUtensorMap* a, const CUtensorMap* b, const GemmEpi& ep, int M,
+                        int N, int K, const FilmTiles& film, cudaStream_t s) {
   const int m_tiles = (M + kBM - 1) / kBM;
   FilmTiles f = film;
   f.y0 = N / BN;
   const int extra_y = film.tiles > 0 ? (film.tiles + m_tiles - 1) / m_tiles : 0;
   dim3 grid(m_tiles, N / BN + extra_y, 1);
-  return launch_pdl(tc_gemm_kernel<BN, GEMM_QKV_ROPE>, grid, dim3(kThreads),
-                    GemmCfg<BN>::kSmemBytes, s, *a, *b, ep, M, N, K / kBK, K / kBK, f);
+  return launch_pdl(tc_gemm_kernel<BN, MODE>, grid, dim3(kThreads), GemmCfg<BN>::kSmemBytes, s,
+                    *a, *b, ep, M, N, K / kBK, K / kBK, f);
+}
+
+bool film_ok(const FilmTiles& film, int K) {
+  if (film.tiles == 0) return true;
+  return film.tiles > 0 && K % kBK == 0 && K / kBK <= kFilmMaxKb &&
+         film.rows >= 1 && film.rows <= kStreamRows && film.tile0 >= 0 &&
+         film.ldo % kFilmTile == 0 && (film.tile0 + film.tiles) * kFilmTile <= film.ldo;
 }
 
 }  // namespace
@@ -718,38 +727,32 @@ cudaError_t launch_tc_gemm_persist(int bn, int mode, const CUtensorMap* a, const
   return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_tc_gemm_qkv_film(int bn, const CUtensorMap* a, const CUtensorMap* b,
-                                    const GemmEpi& ep, int M, int N, int K, const FilmTiles& film,
-                                    cudaStream_t s) {
+cudaError_t launch_tc_gemm_film(int bn, int mode, const CUtensorMap* a, const CUtensorMap* b,
+                                const GemmEpi& ep, int M, int N, int K, const FilmTiles& film,
+                                cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  if (N % bn != 0 || K % kBK != 0 || film.rows > kStreamRows || film.tiles < 0 ||
-      (film.tiles > 0 && K / kBK > FilmCfg<kBnQKV>::kMaxKb) ||
-      film.tile0 < 0 || (film.tiles > 0 && (film.rows < 1 || film.ldo % bn != 0 ||
-                                            (film.tile0 + film.tiles) * bn > film.ldo)))
-    return cudaErrorInvalidValue;
-  if (bn == kBnQKV) return launch_qkv_film<kBnQKV>(a, b, ep, M, N, K, film, s);
-  if (bn == kBnSmall) return launch_qkv_film<kBnSmall>(a, b, ep, M, N, K, film, s);
+  if (N % bn != 0 || K % kBK != 0 || !film_ok(film, K)) return cudaErrorInvalidValue;
+  if (bn == kBnQKV && mode == GEMM_QKV_ROPE)
+    return launch_film<kBnQKV, GEMM_QKV_ROPE>(a, b, ep, M, N, K, film, s);
+  if (bn == kBnSmall && mode == GEMM_QKV_ROPE)
+    return launch_film<kBnSmall, GEMM_QKV_ROPE>(a, b, ep, M, N, K, film, s);
+  if (bn == kBnGU && mode == GEMM_GEGLU)
+    return launch_film<kBnGU, GEMM_GEGLU>(a, b, ep, M, N, K, film, s);
+  if (bn == kBnSmall && mode == GEMM_GEGLU)
+    return launch_film<kBnSmall, GEMM_GEGLU>(a, b, ep, M, N, K, film, s);
   return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_tc_film_tiles(int bn, const FilmTiles& film, int K, int* err, cudaStream_t s) {
+cudaError_t launch_tc_film_tiles(const FilmTiles& film, int K, int* err, cudaStream_t s) {
   if (film.tiles <= 0) return cudaSuccess;
-  if (K % kBK != 0 || K / kBK > FilmCfg<kBnQKV>::kMaxKb || film.rows < 1 ||
-      film.rows > kStreamRows || film.tile0 < 0 || film.ldo % bn != 0 ||
-      (film.tile0 + film.tiles) * bn > film.ldo)
-    return cudaErrorInvalidValue;
+  if (!film_ok(film, K)) return cudaErrorInvalidValue;
   FilmTiles f = film;
   f.y0 = 0;  // every CTA is a FiLM tile
   GemmEpi ep{};
   ep.err = err;
-  const dim3 grid(1, film.tiles, 1);
-  if (bn == kBnQKV)
-    return launch_pdl(tc_gemm_kernel<kBnQKV, GEMM_QKV_ROPE>, grid, dim3(kThreads),
-                      GemmCfg<kBnQKV>::kSmemBytes, s, f.a, f.b, ep, 0, 0, K / kBK, K / kBK, f);
-  if (bn == kBnSmall)
-    return launch_pdl(tc_gemm_kernel<kBnSmall, GEMM_QKV_ROPE>, grid, dim3(kThreads),
-                      GemmCfg<kBnSmall>::kSmemBytes, s, f.a, f.b, ep, 0, 0, K / kBK, K / kBK, f);
-  return cudaErrorInvalidValue;
+  return launch_pdl(tc_gemm_kernel<kBnSmall, GEMM_QKV_ROPE>, dim3(1, film.tiles, 1),
+                    dim3(kThreads), GemmCfg<kBnSmall>::kSmemBytes, s, f.a, f.b, ep, 0, 0, K / kBK,
+                    K / kBK, f);
 }
 
 cudaError_t launch_tc_gemm(int bn, int mode, const CUtensorMap* a, const CUtensorMap* b,

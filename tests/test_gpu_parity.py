@@ -402,7 +402,9 @@ def test_short_a_boxes_bitwise(wl_kw):
     dict(),                                                   # 2 layers, W 256, 3 chunks
     dict(n_layers=6, width=512, mlp_dim=1024, n_chunks=10, chunk_tokens=8, prefix_lens=[200]),
     dict(n_layers=4, n_chunks=4, chunk_tokens=10, batch=2, prefix_lens=[64, 150]),
-], ids=["L2", "L6_K10", "B2_K4"])
+    # 800 rows: the QKV launch leaves too few SMs, the gate/up launch takes the rest
+    dict(n_chunks=8, chunk_tokens=50, batch=2, prefix_lens=[64, 100]),
+], ids=["L2", "L6_K10", "B2_K4", "B2_K8_gate_up"])
 def test_film_overlap_matches_serial_bitwise(wl_kw):
     """FiLM modulation carried by the QKV projections (layer 0's scale / shift pair
     first, then each layer's QKV launch computing the next 6W columns in extra CTAs)
