@@ -10,8 +10,10 @@ tail push.
 Prints ONE JSON line (rank 0):
   value       steps/s with every input resident in HBM (CUDA-graph replay through
               fva_step, CUDA events on the launching stream, max over ranks);
-  e2e         the same through the C ABI with the buffer copied in from pinned host
-              memory and the emitted chunk copied back every step;
+  e2e         the same through the C ABI on pinned host buffers: every step's kernels
+              read the action buffer from host memory and write the updated buffer
+              and the emitted chunk back (e2e_copies: torch copies on the stream
+              around the step on device buffers instead);
   roofline    the dominant kernel (largest share of a kernel-by-kernel profiled
               step) against the measured peak of its binding resource;
   step_roofline  the whole step against max(FLOPs / tensor peak, bytes / HBM peak);
@@ -489,27 +491,48 @@ def main():
     value = steps_total / (ms / 1e3)
     us_per_step = 1e3 * ms / args.steps
 
-    # ---- end to end: pinned host buffer in, emitted chunk out, every step
+    # ---- end to end: the C-ABI step on pinned HOST buffers.  Every step's kernels read
+    # the action buffer from host memory (the in-projection and the Euler update each
+    # read it), write the updated buffer and the emitted chunk back to host memory,
+    # and take tau / dt from the pinned parameter ring: all transfers happen inside
+    # the timed steps, over the host link, with no copy queued on the stream.
     h_buf = torch.from_numpy(buf).pin_memory()
     h_out = torch.empty((B, wl.chunk_tokens, wl.action_dim)).pin_memory()
     e2e_steps = max(10, args.steps // 4)
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
-            d_buf.copy_(h_buf, non_blocking=True)
-            fva.fva_step(h, d_buf, tau, d_out, B, stream)
-            h_out.copy_(d_out, non_blocking=True)
+            fva.fva_step(h, h_buf, tau, h_out, B, stream)
         barrier()
         ev0.record(stream)
         for _ in range(e2e_steps):
-            d_buf.copy_(h_buf, non_blocking=True)
-            fva.fva_step(h, d_buf, tau, d_out, B, stream)
-            h_out.copy_(d_out, non_blocking=True)
+            fva.fva_step(h, h_buf, tau, h_out, B, stream)
         ev1.record(stream)
     barrier()
     e2e_ms = max_over_ranks(ev0.elapsed_time(ev1))
     e2e_value = e2e_steps * world / (e2e_ms / 1e3)
-    h2d = buf.nbytes + tau.nbytes
-    d2h = h_out.numel() * 4
+    h2d = 2 * buf.nbytes + tau.nbytes
+    d2h = buf.nbytes + h_out.numel() * 4
+    # the same through copies queued on the stream around the step on device buffers
+    # (pinned buffer in, emitted chunk out): context for the number above
+    e2e_copies = None
+    if rank == 0:
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                d_buf.copy_(h_buf, non_blocking=True)
+                fva.fva_step(h, d_buf, tau, d_out, B, stream)
+                h_out.copy_(d_out, non_blocking=True)
+            ec0 = torch.cuda.Event(enable_timing=True)
+            ec1 = torch.cuda.Event(enable_timing=True)
+            ec0.record(stream)
+            for _ in range(e2e_steps):
+                d_buf.copy_(h_buf, non_blocking=True)
+                fva.fva_step(h, d_buf, tau, d_out, B, stream)
+                h_out.copy_(d_out, non_blocking=True)
+            ec1.record(stream)
+        torch.cuda.synchronize()
+        e2e_copies = {"value": e2e_steps / (ec0.elapsed_time(ec1) / 1e3), "unit": "steps/s",
+                      "h2d_bytes_per_step": buf.nbytes, "d2h_bytes_per_step": h_out.numel() * 4,
+                      "note": "torch copies on the stream around fva_step on device buffers"}
 
     # ---- the same step reusing the previous step's FiLM modulation (steady streaming
     # keeps the noise levels fixed, §3.2): a separately labelled extra number
@@ -683,7 +706,10 @@ def main():
                 "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": cfg_json,
                 "clocks": clocks,
                 "e2e": {"value": e2e_value, "unit": "steps/s", "h2d_bytes_per_step": h2d,
-                        "d2h_bytes_per_step": d2h, "steps": e2e_steps},
+                        "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+                        "api": "fva_step on pinned host buffers (the step's kernels read and "
+                               "write host memory over the host link)"},
+                "e2e_copies": e2e_copies,
                 "gpu_launches": launches_per_step * args.steps,
                 "roofline": roof, "step_roofline": step_roof, "kernel_shares": shares,
                 "kernel_rooflines": kernel_rooflines,

@@ -201,13 +201,19 @@ fva_status fva_share_prefix_kv(fva_handle* h, int32_t request, int32_t src_reque
 /*
  * One steady-streaming step (§3.2, Algorithm 1; Eq. 1 and 2) for `batch`
  * independent requests, queued on `stream`; returns without waiting.
- *   buffer       device fp32 [batch, K, H, A], slot 0 = cleanest chunk; updated in
- *                place to [x'_2, ..., x'_K, z] where x'_k = x_k + dt_k v_k.
+ *   buffer       fp32 [batch, K, H, A], slot 0 = cleanest chunk; updated in place
+ *                to [x'_2, ..., x'_K, z] where x'_k = x_k + dt_k v_k.
  *   noise_levels host fp32 [batch, K]: tau_1 < ... < tau_K, each in (0, 1], per
  *                request (read before the call returns).  dt_k = tau_{k-1} - tau_k
  *                with tau_0 = 0, computed in fp32.
- *   out_chunk    device fp32 [batch, H, A]: the emitted clean chunk x'_1.
+ *   out_chunk    fp32 [batch, H, A]: the emitted clean chunk x'_1.
  *   batch        1 .. max_batch.
+ * buffer and out_chunk are device memory, or pinned host memory mapped at the same
+ * address (cudaHostAlloc / cudaMallocHost, or cudaHostRegister with the mapped flag,
+ * on a unified-address system): the step's kernels then read the buffer from and
+ * write the buffer and the chunk to host memory themselves, over the host link
+ * (NVLink-C2C on Grace), without a copy on the stream.  Pageable host memory is
+ * refused (INVALID_ARG) before anything is queued.
  * The tail chunk z is drawn from Philox4x32-10 (key noise_seed, counter =
  * (element/4, request, step index)) with Box-Muller; the step index starts at 0 and
  * increases by one per call.  No allocation and no host synchronisation happen

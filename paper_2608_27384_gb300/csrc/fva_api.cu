@@ -1308,6 +1308,28 @@ extern "C" int64_t fva_trace_floats(const fva_handle* h, int32_t batch) {
   return M * (5LL * h->W + 2LL * h->Dq + 2LL * h->dh + h->F) + (int64_t)batch * h->K * h->W;
 }
 
+// A pointer the step's kernels dereference: device memory of the handle's device, or
+// pinned host memory mapped at the same address (the kernels then read and write it
+// over the host link).  Pageable host memory is refused before any launch.
+static fva_status check_step_ptr(fva_handle* h, const void* p, const char* what) {
+  cudaPointerAttributes at{};
+  cudaError_t e = cudaPointerGetAttributes(&at, p);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(FVA_ERR_INVALID_ARG, "%s: cudaPointerGetAttributes failed: %s", what,
+                cudaGetErrorString(e));
+  }
+  const bool device = (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) &&
+                      at.device == h->device;
+  const bool mapped_host = at.type == cudaMemoryTypeHost && at.devicePointer == p;
+  if (!device && !mapped_host)
+    return fail(FVA_ERR_INVALID_ARG,
+                "%s must be memory of device %d or pinned host memory mapped at the same "
+                "address (cudaHostAlloc / cudaHostRegister), not pageable host memory",
+                what, h->device);
+  return FVA_OK;
+}
+
 static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_levels,
                             float* out_chunk, int32_t batch, const fva_step_opts* opts,
                             fva_stream stream, StepProfile* prof) {
@@ -1348,8 +1370,14 @@ static fva_status step_impl(fva_handle* h, float* buffer, const float* noise_lev
     }
   }
   DeviceGuard guard(h->device);
+  fva_status st;
+  if ((st = check_step_ptr(h, buffer, "buffer")) != FVA_OK ||
+      (st = check_step_ptr(h, out_chunk, "out_chunk")) != FVA_OK ||
+      (opts && opts->trace_layer >= 0 &&
+       (st = check_step_ptr(h, opts->trace_out, "trace_out")) != FVA_OK))
+    return st;
   cudaStream_t s = (cudaStream_t)stream;
-  fva_status st = check_async_error(h, s);
+  st = check_async_error(h, s);
   if (st != FVA_OK) return st;
 
   // stage tau, dt and the step index in the next slot of the pinned ring; the

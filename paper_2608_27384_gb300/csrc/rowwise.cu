@@ -141,12 +141,15 @@ __global__ void __launch_bounds__(256) embed_norm_kernel(StepDims d, int rows, c
     for (int a = 0; a < kEmbedMaxA; ++a)
       if (a < d.A) wreg[a] = *reinterpret_cast<const float4*>(w_in_t + (size_t)a * d.W + col);
     const float4 bias = *reinterpret_cast<const float4*>(b_in + col);
-    pdl_trigger();
-    pdl_wait();
+    // the buffer rows were written by the previous step's roll, earlier on the
+    // stream, and by nothing in this step before this kernel: read before the wait
+    // too (from device memory, or from pinned host memory over the host link)
     for (int i = threadIdx.x; i < R * d.A; i += blockDim.x) {
       const int r = i / d.A, a = i % d.A;
       xs[r][a] = r < nr ? buffer[(size_t)(m0 + r) * d.A + a] : 0.f;
     }
+    pdl_trigger();
+    pdl_wait();
     float4 sc[R], sh[R];
 #pragma unroll
     for (int r = 0; r < R; ++r) {
@@ -189,13 +192,14 @@ __global__ void __launch_bounds__(256) embed_norm_kernel(StepDims d, int rows, c
     }
     return;
   }
-  pdl_trigger();
-  pdl_wait();
-  // buffer [B, K, H, A] = rows of A, token rows m0 .. m0 + nr - 1 contiguous
+  // buffer [B, K, H, A] = rows of A, token rows m0 .. m0 + nr - 1 contiguous (read
+  // before the wait, as above)
   for (int i = threadIdx.x; i < R * d.A; i += blockDim.x) {
     const int r = i / d.A, a = i % d.A;
     xs[r][a] = r < nr ? buffer[(size_t)(m0 + r) * d.A + a] : 0.f;
   }
+  pdl_trigger();
+  pdl_wait();
   __syncthreads();
   float ss[R];
 #pragma unroll

@@ -432,6 +432,42 @@ def test_film_overlap_matches_serial_bitwise(wl_kw):
         case.close()
 
 
+def test_host_buffers_step_matches_device_step():
+    """fva_step_ex on pinned host buffers (the step's kernels read the buffer from and
+    write the buffer and the emitted chunk to host memory over the host link) gives
+    the bits of the same steps on device buffers, step after step; pageable host
+    memory is refused before anything is queued."""
+    import torch
+    import paper_2608_27384_gb300 as fva
+    wl = WL.small_bf16_workload(n_chunks=3, prefix_lens=[80])
+    case = Case(wl)
+    try:
+        fresh = case.dev(WL.make_fresh_noise(wl, 1)[0])
+        d_buf = case.dev(case.buf)
+        d_out = torch.empty((1, wl.chunk_tokens, wl.action_dim), device="cuda")
+        h_buf = torch.from_numpy(np.ascontiguousarray(case.buf)).pin_memory()
+        h_out = torch.empty((1, wl.chunk_tokens, wl.action_dim)).pin_memory()
+        base = case.tau.astype(np.float64)
+        for i in range(4):
+            tau = (base * (0.7 + 0.1 * i)).astype(np.float32)
+            fva.fva_step_ex(case.handle, d_buf, tau, d_out, 1, fresh_noise=fresh)
+            fva.fva_step_ex(case.handle, h_buf, tau, h_out, 1, fresh_noise=fresh)
+            torch.cuda.synchronize()
+            for dev_t, host_t, what in ((d_out, h_out, "out"), (d_buf, h_buf, "buffer")):
+                a = dev_t.cpu().numpy()
+                b = host_t.numpy()
+                assert np.isfinite(a).all()
+                assert np.array_equal(a.view(np.uint32), b.view(np.uint32)), (i, what)
+        pageable = torch.from_numpy(np.ascontiguousarray(case.buf))
+        assert not pageable.is_pinned()
+        with pytest.raises(fva.FvaError) as ei:
+            fva.fva_step(case.handle, pageable, case.tau, d_out, 1)
+        assert "INVALID_ARG" in str(ei.value)
+        torch.cuda.synchronize()
+    finally:
+        case.close()
+
+
 def test_step_parameters_follow_every_call():
     """Each step reads its own noise levels through the pinned ring of step
     parameters (8 slots; the step's first kernel copies the slot a device counter
