@@ -1006,6 +1006,7 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
     ft.bias = h->b_mod;
     ft.ldo = h->N_mod;
     ft.rows = BK;
+    ft.pre_stages = 4;
     ft.tile0 = c0 / kFilmTile;
     ft.tiles = n / kFilmTile;
     return ft;
@@ -1044,8 +1045,11 @@ fva_status enqueue_step(fva_handle* h, int B, float* buffer, float* out_chunk, b
       ep.bias = h->b_mod;
       ep.ldo = h->N_mod;
       mark(FVA_K_FILM, -1);
-      if (film_fold)
-        CUDA_TRY(launch_tc_film_tiles(film_tiles(0, 2 * W), W, h->err_dev, s));
+      if (film_fold) {
+        FilmTiles f0 = film_tiles(0, 2 * W);
+        f0.pre_stages = W / 64;  // alone after the time MLP: every stage that fits
+        CUDA_TRY(launch_tc_film_tiles(f0, W, h->err_dev, s));
+      }
       else
         CUDA_TRY(BK <= 16 ? launch_tc_gemm_stream(&h->m_cond16, &h->m_wmod, ep, BK, h->N_mod, W,
                                                   2 * h->n_sms, s)

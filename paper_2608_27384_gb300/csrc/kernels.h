@@ -146,6 +146,7 @@ struct FilmTiles {
   const float* bias;
   int ldo;
   int rows;            // at most 16
+  int pre_stages;      // weight stages requested before the dependency wait (>= 1)
   int tile0, tiles;    // tiles 0: none
   int y0;              // set by the launcher
 };

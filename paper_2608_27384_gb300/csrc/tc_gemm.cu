@@ -102,9 +102,10 @@ __device__ void film_tile_cta(const FilmTiles& fj, uint8_t* smem, uint8_t* bar_a
   pdl_trigger();
 
   if (warp == 0 && lane == 0) {
-    // a few weight stages before the wait (more of them in flight while the
-    // previous kernel runs slowed the step down: 4 measured best on GB300)
-    const int pre = min(nkb, min(F::kStages, 4));
+    // fj.pre_stages weight stages before the wait: inside a projection's launch a
+    // few (more of them in flight while the previous kernel runs slowed the step
+    // down: 4 measured best on GB300), alone all that fit
+    const int pre = min(nkb, min(F::kStages, max(1, fj.pre_stages)));
     for (int i = 0; i < pre; ++i) {
       mbar_arrive_expect_tx(&fullB[i], F::kBBytes);
       tma_load_2d(sB + i * F::kBBytes, &fj.b, i * kBK, n0, &fullB[i]);
