@@ -41,6 +41,23 @@ def test_exports_every_declared_symbol(fva):
         getattr(fva.lib(), name)
 
 
+def test_header_constants_match_binding(fva):
+    """Every integer #define of include/fva.h (flags, ring size, ABI version) has the
+    same value in the Python binding, and every enumerator the binding names exists
+    in the header with that value."""
+    text = open(os.path.join(ROOT, "include", "fva.h")).read()
+    defines = dict((m.group(1), int(m.group(2)))
+                   for m in re.finditer(r"#define (FVA_[A-Z0-9_]+) (\d+)u?\b", text))
+    assert {"FVA_FLAG_NO_GRAPH", "FVA_STEP_REUSE_FILM", "FVA_STEP_SERIAL_FILM",
+            "FVA_PARAM_RING", "FVA_ABI_VERSION"} <= set(defines)
+    for name, value in defines.items():
+        assert getattr(fva, name) == value, name
+    enums = dict((m.group(1), int(m.group(2)))
+                 for m in re.finditer(r"\b(FVA_[A-Z0-9_]+)\s*=\s*(\d+)", text))
+    for name in ("FVA_FP32", "FVA_BF16"):
+        assert getattr(fva, name) == enums[name], name
+
+
 def _cfg(fva, **over):
     wl = WL.standard_workloads()["pi05_2view"]
     from paper_2608_27384_gb300.harness import config_for
